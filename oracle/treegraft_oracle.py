@@ -1,0 +1,254 @@
+"""CPU oracle for TreeGraft's verify-and-grow step (test infrastructure only).
+
+This is a plain, slow statement of what the step computes, written from the
+paper's definitions in fp64 (attention, log-sum-exp) and fp32 (path-score
+sums, whose summation order the definition fixes).  Only the test-suite, the
+package smoke check and the benchmark's CPU-baseline leg may import it; the
+product path never calls it.  It shares no code with the CUDA library: it
+takes plain numpy arrays (bf16 tensors as their uint16 bit patterns) and
+decodes them itself.
+
+Every function is pinned against something other than itself by the
+CPU-only tests in tests/test_oracle_pins.py (brute force, closed forms,
+invariants).  Parity status per function:
+  ancestor_mask, tree_attention, expand_topk, rescore_select, accept:
+  pinned.
+
+Readings of the paper taken here (where it is silent or loose):
+  * depth(root) = 0; mask row u has P + depth(u) + 1 ones (Algorithm 3 mask:
+    root, ancestors, self; plus the whole committed prefix);
+  * every tree node, the root included, has its K/V at cache slot P + node;
+  * scale = D^-1/2, q-head h reads kv-head floor(h / G), G = Hq / Hkv;
+  * edge scores are natural-log probabilities (Sec. 3.1 defines s(v) as a
+    product of probabilities; the log of it is a sum), s(root) = 0;
+  * top-k and Top_W rank by the input value, ties to the lower token / node
+    id;
+  * the stronger drafter rescores a non-root node v from the row of its
+    parent: p(v) = q_m(token(v) | prefix ending at pa(v)) (Sec. 3.1, 3.2);
+  * verification at temperature 0 is greedy matching against the target's
+    argmax (lowest token on ties); the accepted node is the deepest fully
+    matching node, ties to the lowest id; the bonus token is the argmax of
+    the accepted node's own row.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+NEG_INF = float("-inf")
+
+
+def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Decode raw bf16 bit patterns (uint16) exactly into float64."""
+    b = np.ascontiguousarray(bits).view(np.uint16).astype(np.uint32) << 16
+    return b.view(np.float32).astype(np.float64)
+
+
+def _tree_slices(node_off):
+    node_off = np.asarray(node_off, dtype=np.int64)
+    return [(int(node_off[b]), int(node_off[b + 1])) for b in range(len(node_off) - 1)]
+
+
+def check_tree(parent: np.ndarray) -> None:
+    """Raise if a tree's parent array is not in parents-before-children form
+    (Algorithm 3 re-indexes the verification tree so that it is)."""
+    parent = np.asarray(parent)
+    if len(parent) == 0 or parent[0] != -1:
+        raise ValueError("root must be node 0 with parent -1")
+    for i in range(1, len(parent)):
+        if not (0 <= parent[i] < i):
+            raise ValueError(f"parent[{i}] = {parent[i]} is not an earlier node")
+
+
+def node_depth(parent: np.ndarray) -> np.ndarray:
+    """Depth of every node, root depth 0 (position id, Algorithm 3)."""
+    check_tree(parent)
+    d = np.zeros(len(parent), dtype=np.int64)
+    for u in range(len(parent)):
+        v, k = u, 0
+        while parent[v] != -1:
+            v = parent[v]
+            k += 1
+        d[u] = k
+    return d
+
+
+def ancestor_mask(parent: np.ndarray) -> np.ndarray:
+    """Tree-attention mask of Algorithm 3: mask[u, v] is true iff v is the
+    root, an ancestor of u, or u itself.  Computed by walking parent pointers
+    from u up to the root."""
+    check_tree(parent)
+    n = len(parent)
+    m = np.zeros((n, n), dtype=bool)
+    for u in range(n):
+        m[u, 0] = True
+        v = u
+        while v != -1:
+            m[u, v] = True
+            v = int(parent[v])
+    return m
+
+
+def tree_attention(q, k_cache, v_cache, prefix_len, parent, node_off, Hkv: int,
+                   scale: float | None = None, *, bf16: bool = True):
+    """Ancestor-masked GQA tree attention in fp64.
+
+    For tree b, q-head h and node u the keys are the committed prefix
+    [0, P_b) and the tree slots P_b + v of the nodes v allowed by the
+    Algorithm-3 mask of u (root, ancestors, self); the tree is verified
+    through tree attention (Sec. 3.1; Algorithm 1/2 verification step).
+
+      s_j = scale * <q, k_j>,  o = sum_j softmax(s)_j v_j,  lse = log sum_j e^{s_j}
+
+    q: [n_total, Hq, D]; k_cache, v_cache: [B, Hkv, S_max, D] (bf16 bits if
+    bf16 else float arrays).  Returns (o float64 [n_total, Hq, D],
+    lse float64 [n_total, Hq]).
+    """
+    if bf16:
+        q, k_cache, v_cache = (bf16_bits_to_f64(x) for x in (q, k_cache, v_cache))
+    else:
+        q, k_cache, v_cache = (np.asarray(x, dtype=np.float64) for x in (q, k_cache, v_cache))
+    n_total, Hq, D = q.shape
+    G = Hq // Hkv
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    o = np.zeros((n_total, Hq, D))
+    lse = np.zeros((n_total, Hq))
+    for b, (a, e) in enumerate(_tree_slices(node_off)):
+        n, P = e - a, int(prefix_len[b])
+        allowed = np.concatenate([np.ones((n, P), bool), ancestor_mask(parent[a:e])], axis=1)
+        for h in range(Hq):
+            kv = h // G
+            K = k_cache[b, kv, :P + n]
+            Vv = v_cache[b, kv, :P + n]
+            s = (q[a:e, h] @ K.T) * scale
+            s[~allowed] = NEG_INF
+            m = s.max(axis=1, keepdims=True)
+            p = np.exp(s - m)
+            l = p.sum(axis=1, keepdims=True)
+            o[a:e, h] = (p @ Vv) / l
+            lse[a:e, h] = (m + np.log(l))[:, 0]
+    return o, lse
+
+
+def _row_values(logits, r: int, bf16: bool) -> np.ndarray:
+    row = logits[r]
+    return bf16_bits_to_f64(row) if bf16 else np.asarray(row, dtype=np.float64)
+
+
+def expand_topk(logits, parent_score, k: int, row_idx=None, *, bf16: bool = False):
+    """Per-row log-softmax, top-k child tokens and cumulative path score.
+
+    For each logical row i (physical row row_idx[i], or i):
+      lse = log sum_t exp(l_t)                         (fp64)
+      tok = the k tokens of largest l_t, ordered by (l desc, token asc)
+      logprob = fp32(l_tok - lse)       edge score p(u) in log form (Alg. 1/2)
+      score = fp32(parent_score + l_tok - lse)   s(u) = s(v) * p(u) in log form
+    A row whose logits are all -inf has lse = -inf and logprob = score = -inf.
+    Returns tok int32 [rows, k], logprob f32, score f32, lse f64 [rows].
+    """
+    rows = len(parent_score)
+    tok = np.zeros((rows, k), dtype=np.int32)
+    lp = np.zeros((rows, k), dtype=np.float32)
+    sc = np.zeros((rows, k), dtype=np.float32)
+    lse = np.zeros(rows)
+    for i in range(rows):
+        r = int(row_idx[i]) if row_idx is not None else i
+        x = _row_values(logits, r, bf16)
+        V = len(x)
+        m = x.max()
+        if m == NEG_INF:
+            lse[i] = NEG_INF
+        else:
+            lse[i] = m + np.log(np.exp(x - m).sum())
+        order = np.lexsort((np.arange(V), -x))[:k]
+        tok[i] = order
+        if lse[i] == NEG_INF:
+            lp[i] = NEG_INF
+            sc[i] = NEG_INF
+        else:
+            lp[i] = (x[order] - lse[i]).astype(np.float32)
+            sc[i] = (float(np.float32(parent_score[i])) + (x[order] - lse[i])).astype(np.float32)
+    return tok, lp, sc, lse
+
+
+def rescore_select(weak_edge, strong_lp, parent, token, visited, node_off, N: int):
+    """Stronger-drafter rescoring of the candidate pool and global top-N.
+
+    Per tree (Sec. 3.2, Algorithm 2 middle-drafter step): the candidate pool
+    is C = {v : not visited[v]} = V(T) \\ P_k.  For non-root v in C the edge
+    score becomes the stronger drafter's log-prob of token(v) under the
+    prefix ending at pa(v): strong_lp[pa(v), token(v)]; other nodes keep
+    weak_edge[v].  Scores are recomputed as fp32 sums from the root,
+    s(root) = 0, s(v) = fp32(s(pa(v)) + edge(v)) in node order.  The
+    frontier is Top_N(C, s) ordered by (s desc, id asc).
+
+    Returns edge f32 [n_total] (root entries 0), score f32 [n_total],
+    selected int32 [B, N] (local node ids, -1 padded), n_selected int32 [B].
+    """
+    n_total = len(parent)
+    edge = np.zeros(n_total, dtype=np.float32)
+    score = np.zeros(n_total, dtype=np.float32)
+    slices = _tree_slices(node_off)
+    sel = np.full((len(slices), N), -1, dtype=np.int32)
+    nsel = np.zeros(len(slices), dtype=np.int32)
+    for b, (a, e) in enumerate(slices):
+        check_tree(parent[a:e])
+        for v in range(1, e - a):
+            if visited[a + v]:
+                edge[a + v] = np.float32(weak_edge[a + v])
+            else:
+                edge[a + v] = np.float32(strong_lp[a + int(parent[a + v]), int(token[a + v])])
+        score[a] = np.float32(0.0)
+        for v in range(1, e - a):
+            score[a + v] = np.float32(score[a + int(parent[a + v])]) + np.float32(edge[a + v])
+        cand = [v for v in range(e - a) if not visited[a + v]]
+        cand.sort(key=lambda v: (-float(score[a + v]), v))
+        take = cand[:N]
+        sel[b, :len(take)] = take
+        nsel[b] = len(take)
+    return edge, score, sel, nsel
+
+
+def target_argmax(target_logits, rows, *, bf16: bool = False) -> np.ndarray:
+    """Greedy target token per row: argmax with the lowest token on ties."""
+    return np.array([int(np.argmax(_row_values(target_logits, r, bf16))) for r in rows],
+                    dtype=np.int64)
+
+
+def accept(target_logits, token, parent, node_off, path_cap: int, *, bf16: bool = False):
+    """Greedy longest-accepted-path walk at temperature 0 (Sec. 5 setting;
+    the verification step of Algorithms 1 and 2).
+
+    Brute force: enumerate every root-to-node path; a path is accepted when
+    each of its non-root nodes' token equals the target argmax of its
+    parent's row.  The accepted node a* is the deepest fully matching node,
+    ties to the lowest id; A = depth(a*); the bonus token is the argmax of
+    row a*.  Returns path int32 [B, path_cap] (root-first local ids, -1
+    padded), accept_len int32 [B], bonus int32 [B].
+    """
+    slices = _tree_slices(node_off)
+    path = np.full((len(slices), path_cap), -1, dtype=np.int32)
+    alen = np.zeros(len(slices), dtype=np.int32)
+    bonus = np.zeros(len(slices), dtype=np.int32)
+    for b, (a, e) in enumerate(slices):
+        par = parent[a:e]
+        check_tree(par)
+        am = target_argmax(target_logits, range(a, e), bf16=bf16)
+        best = None
+        for v in range(e - a):
+            chain = [v]
+            while par[chain[-1]] != -1:
+                chain.append(int(par[chain[-1]]))
+            chain.reverse()
+            ok = all(int(token[a + w]) == am[int(par[w])] for w in chain[1:])
+            if ok:
+                key = (len(chain) - 1, -v)
+                if best is None or key > best[0]:
+                    best = (key, chain)
+        chain = best[1]
+        if len(chain) > path_cap:
+            raise ValueError("accepted path longer than path_cap")
+        path[b, :len(chain)] = chain
+        alen[b] = len(chain) - 1
+        bonus[b] = am[chain[-1]]
+    return path, alen, bonus
