@@ -1,0 +1,548 @@
+#!/usr/bin/env python
+"""Benchmark of the TreeGraft verify-and-grow step on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input
+of the Llama-3-8B-shaped verify workload (batch 1, prefix 2048, 60-node tree
+of depth 6, GQA 32/8, head_dim 128, vocab 128256, bf16):
+  treegraft_tree_attn      target verification attention over prefix + tree
+  treegraft_expand_topk    per-node log-softmax + top-10 + path scores (drafter rows)
+  treegraft_rescore_select stronger-drafter rescoring + top-10 reselection
+  treegraft_accept         greedy longest accepted path on the target rows
+
+Inputs are resident in HBM; eight input sets are rotated so that the bytes
+touched between two uses of a set (~280 MB) exceed the 126 MB L2.  Steps
+are replayed from CUDA graphs.  Per-kernel durations come from graphs of
+that kernel alone, timed with CUDA events on the launching stream.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun (N > 1) every rank runs its own independent sequences (the
+verify step of one sequence never needs another's data): weak scaling, no
+data-path collective; the barrier and the max-over-ranks time use NCCL.
+Rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "tree-verify steps/s & tree_attn HBM GB/s (% of peak), Llama-3-8B shape"
+WORKLOAD = "llama3-8b-verify"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20000)
+    p.add_argument("--warmup", type=int, default=50)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--sets", type=int, default=8)
+    p.add_argument("--seed", type=int, default=0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+# --------------------------------------------------------------------------- workload
+
+def algorithmic_costs(wl):
+    """Bytes each call must move at minimum and the attention FLOPs."""
+    sh = wl["shape"]
+    n = len(wl["parent"])
+    P = int(wl["prefix_len"][0])
+    Hq, Hkv, D, V, k, N = sh["Hq"], sh["Hkv"], sh["D"], sh["V"], sh["k"], sh["N"]
+    depth = [0] * n
+    for v in range(1, n):
+        depth[v] = depth[wl["parent"][v]] + 1
+    keys = sum(P + d + 1 for d in depth)
+    attn_bytes = 2 * (P + n) * Hkv * D * 2 + 2 * n * Hq * D * 2 + n * 4 * 2
+    attn_flops = 4 * Hq * D * keys
+    expand_bytes = n * V * 2 + n * 4 + n * k * 12
+    accept_bytes = n * V * 2 + n * 8 + 4 * 3 + n * 4
+    rescore_bytes = n * (4 + 4 + 4 + 4 + 1) + n * 4 + n * 8 + N * 4
+    return dict(tree_attn=(attn_bytes, attn_flops), expand_topk=(expand_bytes, 0),
+                rescore_select=(rescore_bytes, 0), accept=(accept_bytes, 0))
+
+
+def build_sets(R, seed, dev):
+    import numpy as np
+    import torch
+    from paper_2608_26112_gb300 import synth
+
+    def bf(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    def t(a):
+        return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+    sets, host = [], []
+    for r in range(R):
+        wl = synth.make_workload(WORKLOAD, seed=seed + r, with_strong=(r == 0))
+        rng = synth.make_rng(10_000 + seed + r)
+        # target rows for accept: a second, independent logit array with its own bumps
+        tl = synth.normal_f32(rng, wl["logits"].shape, 3.0)
+        synth.plant_child_bump(rng, tl, wl["parent"], wl["token"], np.arange(len(wl["parent"])))
+        wl["target_logits"] = synth.f32_to_bf16_bits(tl)
+        if r == 0:
+            strong = t(wl["strong_lp"])
+        d = dict(q=bf(wl["q"]), k=bf(wl["k_cache"]), v=bf(wl["v_cache"]),
+                 prefix_len=t(wl["prefix_len"]), parent=t(wl["parent"]), token=t(wl["token"]),
+                 node_off=t(wl["node_off"]), logits=bf(wl["logits"]),
+                 target=bf(wl["target_logits"]), parent_score=t(wl["parent_score"]),
+                 weak_edge=t(wl["weak_edge"]), visited=t(wl["visited"]), strong=strong)
+        sets.append(d)
+        wl.pop("strong_lp", None)
+        host.append(wl)
+    return sets, host
+
+
+def alloc_outputs(d, sh, dev):
+    import torch
+    import paper_2608_26112_gb300 as tg
+    n = d["parent"].shape[0]
+    k, N = sh["k"], sh["N"]
+    return dict(
+        o=torch.empty_like(d["q"]),
+        tok=torch.empty(n, k, dtype=torch.int32, device=dev),
+        lp=torch.empty(n, k, dtype=torch.float32, device=dev),
+        sc=torch.empty(n, k, dtype=torch.float32, device=dev),
+        edge=torch.empty(n, dtype=torch.float32, device=dev),
+        score=torch.empty(n, dtype=torch.float32, device=dev),
+        sel=torch.empty(1, N, dtype=torch.int32, device=dev),
+        nsel=torch.empty(1, dtype=torch.int32, device=dev),
+        path=torch.empty(1, n, dtype=torch.int32, device=dev),
+        alen=torch.empty(1, dtype=torch.int32, device=dev),
+        bonus=torch.empty(1, dtype=torch.int32, device=dev),
+        ws=tg.accept_workspace(1, n, dev))
+
+
+def call(name, d, o, sh):
+    import paper_2608_26112_gb300 as tg
+    n = d["parent"].shape[0]
+    if name == "tree_attn":
+        tg.tree_attn(d["q"], d["k"], d["v"], d["prefix_len"], d["parent"], d["node_off"], n,
+                     out=o["o"])
+    elif name == "expand_topk":
+        tg.expand_topk(d["logits"], d["parent_score"], sh["k"], out=(o["tok"], o["lp"], o["sc"]))
+    elif name == "rescore_select":
+        tg.rescore_select(d["weak_edge"], d["strong"], d["parent"], d["token"], d["visited"],
+                          d["node_off"], n, sh["N"],
+                          out=(o["edge"], o["score"], o["sel"], o["nsel"]))
+    elif name == "accept":
+        tg.accept(d["target"], d["token"], d["parent"], d["node_off"], n, n, o["ws"],
+                  out=(o["path"], o["alen"], o["bonus"]))
+
+
+KERNELS = ["tree_attn", "expand_topk", "rescore_select", "accept"]
+
+
+def step(d, o, sh):
+    for name in KERNELS:
+        call(name, d, o, sh)
+
+
+def capture(fn, stream):
+    import torch
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    return g
+
+
+def time_graph(g, reps, stream):
+    import torch
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    e1.synchronize()
+    return e0.elapsed_time(e1) / 1e3  # seconds
+
+
+# --------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev_index):
+        self.proc = None
+        self.dev_index = dev_index
+
+    def __enter__(self):
+        import torch
+        sel = str(self.dev_index)
+        try:
+            u = str(torch.cuda.get_device_properties(self.dev_index).uuid)
+            sel = u if u.startswith("GPU-") else "GPU-" + u
+        except Exception:
+            pass
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50", "-i", sel], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                text=True)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            time.sleep(0.1)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out = ""
+            self.lines = [ln for ln in out.splitlines() if ln.strip()]
+
+    def summary(self):
+        rows = []
+        for ln in getattr(self, "lines", []):
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(parts[1]), smax=float(parts[2]), power=float(parts[3]),
+                                 hw=parts[5], hwt=parts[6], swt=parts[7], swp=parts[8]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        load = [r for r in rows if r["power"] > 0] or rows
+        reasons = set()
+        for r in load:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("swp", "sw_power_cap")):
+                if r[key].lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in load),
+                "sm_max_mhz": max(r["smax"] for r in load), "reasons": sorted(reasons),
+                "samples": len(load), "power_w_max": max(r["power"] for r in load)}
+
+
+# --------------------------------------------------------------------------- CPU baseline
+
+CPU_SNIPPET = r"""
+import json, sys, time
+sys.path.insert(0, {root!r})
+import numpy as np
+from oracle import treegraft_oracle as O
+from paper_2608_26112_gb300 import synth
+wl = synth.make_workload({workload!r}, seed=0)
+sh = wl["shape"]; n = len(wl["parent"])
+def one_step():
+    O.tree_attention(wl["q"], wl["k_cache"], wl["v_cache"], wl["prefix_len"], wl["parent"],
+                     wl["node_off"], Hkv=sh["Hkv"])
+    O.expand_topk(wl["logits"], wl["parent_score"], sh["k"], bf16=True)
+    O.rescore_select(wl["weak_edge"], wl["strong_lp"], wl["parent"], wl["token"], wl["visited"],
+                     wl["node_off"], sh["N"])
+    O.accept(wl["logits"], wl["token"], wl["parent"], wl["node_off"], n, bf16=True)
+for _ in range({warmup}):
+    one_step()
+t0 = time.perf_counter(); k = 0
+while True:
+    one_step(); k += 1
+    el = time.perf_counter() - t0
+    if (k >= {steps} and el >= {min_s}) or el >= {max_s}:
+        break
+print(json.dumps(dict(steps=k, seconds=el)))
+"""
+
+
+def run_cpu_oracle(steps, warmup, min_s, max_s):
+    env = dict(os.environ)
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[v] = "1"
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    code = CPU_SNIPPET.format(root=ROOT, workload=WORKLOAD, steps=steps, warmup=warmup,
+                              min_s=min_s, max_s=max_s)
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
+                       timeout=max_s * 3 + 300)
+    if r.returncode != 0:
+        raise RuntimeError("CPU oracle failed: " + r.stderr[-2000:])
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    return d["steps"], d["seconds"]
+
+
+# --------------------------------------------------------------------------- traffic record
+
+def traffic_record(kernel):
+    """dram read+write bytes per launch from the committed ncu summary, or
+    None if the kernel's source changed since those counters were taken."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        rec = json.load(f).get(kernel)
+    if not rec:
+        return None
+    src = os.path.join(ROOT, "paper_2608_26112_gb300", "csrc", rec["source"])
+    with open(src, "rb") as f:
+        h = hashlib.sha256(f.read()).hexdigest()[:16]
+    return rec["bytes_per_launch"] if h == rec.get("source_sha256_16") else None
+
+
+# --------------------------------------------------------------------------- arms
+
+def dist_setup(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return world, rank, local
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+
+
+def reference_arm(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    per_step_min = 0.0
+    steps, sec = run_cpu_oracle(max(1, args.steps if args.steps < 50 else 5),
+                                min(args.warmup, 1), per_step_min, 120.0)
+    v = steps / sec
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "steps/s",
+            "n_gpus": args.gpus, "steps": steps, "warmup": min(args.warmup, 1),
+            "ms_per_step": 1e3 * sec / steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "note": "oracle (plain fp64 numpy) on host cores"},
+            "cpu_baseline": {"value": v, "unit": "steps/s", "cores": 1, "kind": "oracle",
+                             "sample": f"{steps} full steps of {WORKLOAD}"},
+            "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def ours_arm(args):
+    import numpy as np
+    import torch
+
+    world, rank, local = dist_setup(args)
+    from paper_2608_26112_gb300 import build as _b
+    if rank == 0:
+        _b.build()
+    if world > 1:
+        barrier(world)
+    import paper_2608_26112_gb300 as tg
+    from paper_2608_26112_gb300 import synth
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    R = args.sets
+    sets, host = build_sets(R, args.seed + 1000 * rank, dev)
+    sh = host[0]["shape"]
+    outs = [alloc_outputs(d, sh, dev) for d in sets]
+    stream = torch.cuda.Stream(device=dev)
+
+    # warm-up through the plain API (also initialises the library's caches)
+    with torch.cuda.stream(stream):
+        for i in range(max(3, args.warmup)):
+            step(sets[i % R], outs[i % R], sh)
+    stream.synchronize()
+    assert tg.last_device_status(stream) == 0
+
+    cycle = capture(lambda: [step(sets[r], outs[r], sh) for r in range(R)], stream)
+    singles = [capture(lambda r=r: step(sets[r], outs[r], sh), stream) for r in range(R)]
+    per_kernel_graphs = {name: capture(lambda name=name: [call(name, sets[r], outs[r], sh)
+                                                         for r in range(R)], stream)
+                         for name in KERNELS}
+    for _ in range(3):
+        cycle.replay()
+    torch.cuda.synchronize()
+
+    K, W = args.steps, args.warmup
+    q, rem = divmod(K, R)
+    clocks = ClockSampler(dev.index)
+    with clocks:
+        # ---- timed region: exactly K steps
+        barrier(world)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(q):
+                cycle.replay()
+            for r in range(rem):
+                singles[r].replay()
+            e1.record(stream)
+        e1.synchronize()
+        barrier(world)
+        t_steps = e0.elapsed_time(e1) / 1e3
+        # ---- per-kernel launch durations (each graph = R launches over the R sets)
+        kreps = max(20, min(2000, int(0.25 / max(1e-6, t_steps / max(1, K)) / R)))
+        kt = {}
+        for name, g in per_kernel_graphs.items():
+            g.replay()
+            kt[name] = time_graph(g, kreps, stream) / (kreps * R)
+    assert tg.last_device_status(stream) == 0
+    t_max = max_over_ranks(t_steps, world)
+    steps_per_s = world * K / t_max
+
+    pk, pk_src = peaks()
+    hbm = pk["hbm_gbs"]
+    costs = algorithmic_costs(host[0])
+    kernels = {}
+    for name in KERNELS:
+        b, f = costs[name]
+        kernels[name] = {"us": kt[name] * 1e6, "bytes": b, "GBps": b / kt[name] / 1e9,
+                         "hbm_frac": b / kt[name] / 1e9 / hbm}
+        if f:
+            kernels[name]["TFLOPs"] = f / kt[name] / 1e12
+    dom = max(KERNELS, key=lambda n: kt[n])
+    b, f = costs[dom]
+    achieved = b / kt[dom] / 1e9
+    roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "traffic": traffic_record(dom),
+                "peak_source": f"{pk_src} hbm_gbs (burst copy)",
+                "algorithmic_bytes_per_launch": b}
+    attn_b, attn_f = costs["tree_attn"]
+    t_attn = kt["tree_attn"]
+    roof_t = max(attn_b / (hbm * 1e9), attn_f / (pk["bf16_tflops"] * 1e12))
+    kernels["tree_attn"]["roofline_frac"] = roof_t / t_attn
+    kernels["tree_attn"]["roofline_frac_8TBps_nominal"] = max(attn_b / 8e12, attn_f / (pk["bf16_tflops"] * 1e12)) / t_attn
+
+    # ---- end to end through the public API with host buffers
+    e2e = end_to_end(host, sh, dev, stream, reps=max(20, min(200, K // 10 or 20)))
+
+    line = {"metric": METRIC, "value": steps_per_s, "unit": "steps/s", "n_gpus": world,
+            "steps": K, "warmup": W, "ms_per_step": 1e3 * t_max / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "batch": 1, "prefix": int(host[0]["prefix_len"][0]),
+                       "tree_nodes": len(host[0]["parent"]), "tree_depth": sh["depth"],
+                       "heads_q_kv": f"{sh['Hq']}/{sh['Hkv']}", "head_dim": sh["D"],
+                       "vocab": sh["V"], "topk": sh["k"], "reselect_N": sh["N"],
+                       "l2": f"{R} rotating input sets, ~{R * 40} MB touched per cycle > 126 MB L2",
+                       "parallelism": f"independent sequences per GPU x{world}"},
+            "roofline": roofline, "kernels": kernels, "e2e": e2e,
+            "gpu_launches": K * len(KERNELS), "clocks": clocks.summary()}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        steps_c, sec = run_cpu_oracle(3, 1, 10.0, 30.0)
+        line["cpu_baseline"] = {"value": steps_c / sec, "unit": "steps/s", "cores": 1,
+                                "kind": "oracle",
+                                "sample": f"{steps_c} full steps of {WORKLOAD} (single thread)"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def end_to_end(host, sh, dev, stream, reps):
+    """Steps/s through the public API with inputs copied from pinned host
+    memory every step and the step's results read back."""
+    import numpy as np
+    import torch
+    import paper_2608_26112_gb300 as tg
+
+    wl = host[0]
+    n = len(wl["parent"])
+
+    def pin(a, dtype=None):
+        t = torch.from_numpy(np.ascontiguousarray(a))
+        if dtype is not None:
+            t = t.view(dtype)
+        return t.pin_memory()
+
+    rng = synth_rng = None
+    hs = dict(q=pin(wl["q"].view(np.int16), torch.bfloat16),
+              k=pin(wl["k_cache"].view(np.int16), torch.bfloat16),
+              v=pin(wl["v_cache"].view(np.int16), torch.bfloat16),
+              prefix_len=pin(wl["prefix_len"]), parent=pin(wl["parent"]), token=pin(wl["token"]),
+              node_off=pin(wl["node_off"]), logits=pin(wl["logits"].view(np.int16), torch.bfloat16),
+              target=pin(wl["target_logits"].view(np.int16), torch.bfloat16),
+              parent_score=pin(wl["parent_score"]), weak_edge=pin(wl["weak_edge"]),
+              visited=pin(wl["visited"]))
+    from paper_2608_26112_gb300 import synth
+    strong_h = pin(synth.make_workload(WORKLOAD, seed=0, with_logits=False)["strong_lp"])
+    hs["strong"] = strong_h
+    d = {k: torch.empty(v.shape, dtype=v.dtype, device=dev) for k, v in hs.items()}
+    o = alloc_outputs(d, sh, dev)
+    res_names = ["o", "tok", "lp", "sc", "edge", "score", "sel", "nsel", "path", "alen", "bonus"]
+    res_h = {k: torch.empty(o[k].shape, dtype=o[k].dtype).pin_memory() for k in res_names}
+    h2d = sum(v.numel() * v.element_size() for v in hs.values())
+    d2h = sum(v.numel() * v.element_size() for v in res_h.values())
+
+    def one():
+        for k_, v in hs.items():
+            d[k_].copy_(v, non_blocking=True)
+        step(d, o, sh)
+        for k_ in res_names:
+            res_h[k_].copy_(o[k_], non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            one()
+    stream.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(reps):
+            one()
+        e1.record(stream)
+    e1.synchronize()
+    t = e0.elapsed_time(e1) / 1e3
+    return {"value": reps / t, "unit": "steps/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": reps}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        ours_arm(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,207 @@
+/*
+ * treegraft.h - C ABI of the GB300 (sm_103a) library for the draft-tree
+ * verify-and-grow step of TreeGraft (multi-drafter tree speculative decoding).
+ *
+ * General contract (all entry points):
+ *  - Every pointer argument is a DEVICE pointer owned by the caller, unless
+ *    stated otherwise.  The library never allocates device memory in these
+ *    calls and never keeps a pointer after the call returns.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Work is enqueued asynchronously on it; the call returns once
+ *    the kernels are launched.
+ *  - Arguments are validated on the host before anything is launched; an
+ *    invalid call returns TG_ERR_INVALID_ARG or TG_ERR_UNSUPPORTED and
+ *    launches nothing.  A failed launch returns TG_ERR_CUDA.
+ *  - Conditions only visible on the device (a malformed parent[] array, a
+ *    bounded wait that gave up) set bits in a per-device status word and the
+ *    kernel returns early without touching memory out of range; read and
+ *    clear that word with treegraft_last_device_status().
+ *  - Trees are batched.  node_off[B+1] (int32) gives tree b the global node
+ *    rows [node_off[b], node_off[b+1]); inside a tree, parent[] holds LOCAL
+ *    ids with parent[0] = -1 and 0 <= parent[i] < i (parents before
+ *    children, the order Algorithm 3 re-indexes the verification tree into).
+ *    Every tree has at least one node (its root) and at most 256 nodes.
+ *  - bf16 data is IEEE bfloat16 (raw 16-bit patterns); all fp32/int32 data
+ *    is native-endian.
+ */
+#ifndef TREEGRAFT_H
+#define TREEGRAFT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  TG_OK = 0,
+  TG_ERR_INVALID_ARG = 1,  /* null pointer, negative or inconsistent size */
+  TG_ERR_UNSUPPORTED = 2,  /* valid but outside what the kernels implement */
+  TG_ERR_CUDA = 3,         /* a CUDA runtime / driver call failed */
+  TG_ERR_DEVICE_TREE = 4,  /* status bit: malformed tree seen on the device */
+  TG_ERR_TIMEOUT = 8,      /* status bit: a bounded device wait gave up */
+  TG_ERR_DEVICE_INDEX = 16 /* status bit: an index read from device memory was out of range */
+} tg_status;
+
+typedef enum { TG_BF16 = 0, TG_F32 = 1 } tg_dtype;
+
+#define TG_MAX_TREE_NODES 256
+#define TG_MAX_TOPK 32
+
+/*
+ * treegraft_tree_attn - ancestor-masked GQA tree attention.
+ *
+ * Paper: every draft-tree node attends over the committed prefix and its own
+ * ancestors (Sec. 3.1 "verified efficiently ... through tree attention";
+ * Algorithm 3 tree-attention mask: mask(u,v)=1 iff v is the root, an
+ * ancestor of u, or u itself).  Used by the target's verification pass and
+ * by the drafters' forward passes over the tree (Algorithms 1 and 2).
+ *
+ * For tree b, q-head h (kv-head h / G, G = Hq / Hkv) and local node u:
+ *   keys J(u) = {0 .. P_b-1} U {P_b + v : mask(u, v)}
+ *   o[u,h] = sum_{j in J(u)} softmax_j(scale * q[u,h] . k[j]) v[j]
+ *   lse[u,h] = log sum_{j in J(u)} exp(scale * q[u,h] . k[j])   (natural log)
+ *
+ * q        bf16 [n_total, Hq, D], row-major (node, head, dim); 16-byte aligned.
+ * k_cache,
+ * v_cache  bf16 [B, Hkv, S_max, D]; slots [0, P_b) hold the committed prefix
+ *          of sequence b, slots [P_b, P_b + n_b) the K/V of the tree's nodes
+ *          in local node order (RoPE already applied by the caller).  Slots
+ *          past P_b + n_b are never used and may hold anything (even NaN).
+ * prefix_len int32 [B] (P_b >= 0, P_b + n_b <= S_max).
+ * parent   int32 [n_total] local parent ids;  node_off int32 [B+1].
+ * max_nodes  upper bound on n_b (<= 256); n_total = total node count.
+ * D in {64, 128}; Hq % Hkv == 0, G = Hq / Hkv in {1, 2, 4, 8}.
+ * scale    softmax scale; 0 selects D^-1/2.
+ * out      bf16 [n_total, Hq, D];  lse_out fp32 [n_total, Hq] or NULL.
+ * Errors: TG_ERR_INVALID_ARG (null pointer, bad sizes, misaligned q/k/v),
+ *   TG_ERR_UNSUPPORTED (D or G outside the list), TG_ERR_CUDA.  A malformed
+ *   tree sets TG_ERR_DEVICE_TREE; its rows of `out` are then left unwritten.
+ */
+int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
+                        const int32_t* prefix_len, const int32_t* parent,
+                        const int32_t* node_off, int B, int max_nodes, int n_total,
+                        int Hq, int Hkv, int D, int S_max, float scale,
+                        void* out, float* lse_out, void* stream);
+
+/*
+ * treegraft_expand_topk - per-node log-softmax, top-k children, path scores.
+ *
+ * Paper: Top_m(l(v)) child tokens of a frontier node, edge score
+ * p(u) = q(y | pi(v)) and cumulative score s(u) = s(v) p(u) (Sec. 3.1;
+ * Algorithm 1, Algorithm 2 small and middle steps), kept in natural-log form.
+ *
+ * For logical row i (physical row r = row_idx ? row_idx[i] : i):
+ *   lse[i]  = log sum_t exp(logits[r, t])
+ *   tok[i,:] = the k token ids with the largest logits[r, t], ordered by
+ *              (logit desc, token id asc) - exact on the input values
+ *   logprob[i,j] = logits[r, tok[i,j]] - lse[i]
+ *   score[i,j]   = parent_score[i] + logprob[i,j]
+ * A row whose logits are all -inf gets lse = logprob = score = -inf and the
+ * k lowest token ids.  Logits must be finite or -inf.
+ *
+ * logits   [logit_rows, ld] elements of `dtype` (TG_BF16 or TG_F32), row r
+ *          at logits + r * ld; V <= ld; V <= 262144 (bf16) or 131072 (fp32).
+ * rows     number of logical rows (rows == 0 is a no-op).
+ * row_idx  int32 [rows] of physical rows in [0, logit_rows), or NULL for
+ *          rows 0..rows-1 (then rows <= logit_rows).
+ * parent_score fp32 [rows].  1 <= k <= min(V, 32).
+ * tok int32 [rows, k], logprob fp32 [rows, k], score fp32 [rows, k],
+ * lse_out fp32 [rows] or NULL.
+ * Errors: TG_ERR_INVALID_ARG, TG_ERR_UNSUPPORTED (V or k too large),
+ *   TG_ERR_CUDA; an out-of-range row_idx sets TG_ERR_DEVICE_INDEX and that
+ *   row's outputs are left unwritten.
+ */
+int treegraft_expand_topk(const void* logits, int dtype, int logit_rows, int V, int64_t ld,
+                          int rows, const int32_t* row_idx, const float* parent_score, int k,
+                          int32_t* tok, float* logprob, float* score, float* lse_out,
+                          void* stream);
+
+/*
+ * treegraft_rescore_select - stronger-drafter rescoring + global top-N.
+ *
+ * Paper: at a middle-drafter step the candidate pool is
+ * C_k = V(T_k) \ P_k (Sec. 3.2, expanded grafting-position selection); for
+ * each non-root v in C_k the middle drafter replaces the edge score p(v),
+ * s(root) stays 1 and s is recomputed; the grafting frontier is
+ * F_k = Top_W(C_k, s) (Algorithm 2, middle-drafter branch).
+ *
+ * Per tree, with local ids and log-domain scores:
+ *   edge[v]  = strong_lp[pa(v), token[v]]   if v != 0 and !visited[v]
+ *            = weak_edge[v]                 if v != 0 and visited[v]
+ *            = 0                            for the root
+ *   score[0] = 0;  score[v] = fp32(score[pa(v)] + edge[v])   (in that order)
+ *   selected = the N nodes of {v : !visited[v]} with the largest score,
+ *              ordered by (score desc, node id asc); n_selected = their count
+ *              (< N when the pool is smaller), remaining slots -1.
+ * weak_edge fp32 [n_total]: stored edge log-probs p(v).
+ * strong_lp fp32 [n_total, ld]: the stronger drafter's next-token log-probs;
+ *   row node_off[b] + v is the distribution after local node v.  V <= ld.
+ * parent, token int32 [n_total]; visited uint8 [n_total] (P_k, non-zero =
+ * visited); node_off int32 [B+1].  1 <= N <= 256.
+ * edge_out, score_out fp32 [n_total]; selected int32 [B, N] (local ids);
+ * n_selected int32 [B].
+ * Errors: TG_ERR_INVALID_ARG, TG_ERR_CUDA; malformed tree or token outside
+ *   [0, V) sets TG_ERR_DEVICE_TREE / TG_ERR_DEVICE_INDEX and that tree's
+ *   outputs are left unwritten.
+ */
+int treegraft_rescore_select(const float* weak_edge, const float* strong_lp, int V, int64_t ld,
+                             const int32_t* parent, const int32_t* token,
+                             const uint8_t* visited, const int32_t* node_off, int B,
+                             int max_nodes, int n_total, int N, float* edge_out,
+                             float* score_out, int32_t* selected, int32_t* n_selected,
+                             void* stream);
+
+/*
+ * treegraft_accept_workspace_size - bytes of scratch treegraft_accept needs.
+ */
+size_t treegraft_accept_workspace_size(int B, int n_total);
+
+/*
+ * treegraft_accept - greedy longest-accepted-path walk (temperature 0).
+ *
+ * Paper: verification of the pruned tree with the target model and the
+ * standard rule (Algorithm 1/2, final step; Sec. 3.2 "Distribution
+ * preservation"), at temperature 0 (Appendix E) - greedy matching.
+ *
+ * Per tree:  am[v] = argmax_t target[v, t] (lowest t on ties);
+ *   full[0] = true; full[v] = full[pa(v)] and token[v] == am[pa(v)];
+ *   a* = the full node of greatest depth, lowest id on ties;
+ *   accept_len = depth(a*) (accepted draft tokens, root excluded);
+ *   path = root-first local ids of the root..a* chain, padded with -1 to
+ *   path_cap; bonus = am[a*] (the target's next token after a*).
+ * target_logits [n_total, ld] of `dtype`; row node_off[b] + v belongs to
+ * local node v.  token int32 [n_total] (token[root] ignored).
+ * path int32 [B, path_cap] (path_cap >= 1); accept_len, bonus int32 [B].
+ * ws       scratch of treegraft_accept_workspace_size(B, n_total) bytes,
+ *          16-byte aligned, ZERO-FILLED before its first use with this
+ *          function; each call leaves it ready for the next call.  Calls
+ *          sharing one ws must not overlap on the GPU.
+ * Errors: TG_ERR_INVALID_ARG, TG_ERR_UNSUPPORTED (V > 262144 for bf16 or
+ *   > 131072 for fp32), TG_ERR_CUDA;
+ *   a malformed tree sets TG_ERR_DEVICE_TREE, a path longer than path_cap
+ *   sets TG_ERR_DEVICE_INDEX (that tree's outputs are then left unwritten).
+ */
+int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld,
+                     const int32_t* token, const int32_t* parent, const int32_t* node_off,
+                     int B, int max_nodes, int n_total, int path_cap, int32_t* path,
+                     int32_t* accept_len, int32_t* bonus, void* ws, size_t ws_bytes,
+                     void* stream);
+
+/*
+ * treegraft_last_device_status - synchronise `stream`, return the OR of the
+ * device status bits raised since the last call on the current device
+ * (TG_OK if none), and clear them.  Returns TG_ERR_CUDA if the
+ * synchronisation itself fails.
+ */
+int treegraft_last_device_status(void* stream);
+
+/* Human-readable name of a status value (static string). */
+const char* treegraft_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TREEGRAFT_H */

@@ -1,0 +1,10 @@
+"""GB300 (sm_103a) kernels for the draft-tree verify-and-grow step of
+TreeGraft (multi-drafter tree speculative decoding).
+
+The compute lives in libtreegraft.so (C ABI, include/treegraft.h); this
+package holds its build script, its Python binding and the seeded synthetic
+input generator used by the tests and the benchmark.
+"""
+from .binding import (  # noqa: F401
+    MAX_TOPK, MAX_TREE_NODES, TreeGraftError, accept, accept_workspace, accept_workspace_size,
+    expand_topk, last_device_status, lib, rescore_select, tree_attn)

@@ -1,0 +1,229 @@
+"""Python binding of libtreegraft.so (the C ABI in include/treegraft.h).
+
+Argument marshalling only: each wrapper checks the torch tensors it is
+given, passes their device pointers and the current CUDA stream to the C
+entry point of the same name, and turns a non-zero status into an
+exception.  Every step of the computation runs in the library's kernels;
+there is no CPU fallback, and a missing library is an error.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libtreegraft.so")
+
+TG_OK = 0
+TG_BF16, TG_F32 = 0, 1
+MAX_TREE_NODES = 256
+MAX_TOPK = 32
+
+_lib = None
+
+
+class TreeGraftError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        msg = lib().treegraft_status_string(status).decode() if _lib else str(status)
+        super().__init__(f"{fn} returned status {status} ({msg})")
+        self.status = status
+
+
+_c_int, _c_i64, _c_f32, _c_vp, _c_size = (ctypes.c_int, ctypes.c_int64, ctypes.c_float,
+                                          ctypes.c_void_p, ctypes.c_size_t)
+
+_SIGNATURES = {
+    "treegraft_tree_attn": [_c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_int, _c_int, _c_int,
+                            _c_int, _c_int, _c_int, _c_int, _c_f32, _c_vp, _c_vp, _c_vp],
+    "treegraft_expand_topk": [_c_vp, _c_int, _c_int, _c_int, _c_i64, _c_int, _c_vp, _c_vp,
+                              _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp],
+    "treegraft_rescore_select": [_c_vp, _c_vp, _c_int, _c_i64, _c_vp, _c_vp, _c_vp, _c_vp,
+                                 _c_int, _c_int, _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp,
+                                 _c_vp],
+    "treegraft_accept_workspace_size": [_c_int, _c_int],
+    "treegraft_accept": [_c_vp, _c_int, _c_int, _c_i64, _c_vp, _c_vp, _c_vp, _c_int, _c_int,
+                         _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_size, _c_vp],
+    "treegraft_last_device_status": [_c_vp],
+    "treegraft_status_string": [_c_int],
+}
+_RESTYPES = {"treegraft_accept_workspace_size": _c_size,
+             "treegraft_status_string": ctypes.c_char_p}
+
+
+def lib() -> ctypes.CDLL:
+    """Load libtreegraft.so (built by paper_2608_26112_gb300.build)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                f"{LIB_PATH} is missing: build it with "
+                "`python -m paper_2608_26112_gb300.build` (nvcc, sm_103a)")
+        dll = ctypes.CDLL(LIB_PATH)
+        for name, argt in _SIGNATURES.items():
+            fn = getattr(dll, name)
+            fn.argtypes = argt
+            fn.restype = _RESTYPES.get(name, _c_int)
+        _lib = dll
+    return _lib
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(fn: str, st: int):
+    if st != TG_OK:
+        raise TreeGraftError(fn, st)
+
+
+def _need(t, dtype, name, device=True):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if device and not t.is_cuda:
+        raise ValueError(f"{name} must live on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def _logit_dtype(t):
+    if t.dtype == torch.bfloat16:
+        return TG_BF16
+    if t.dtype == torch.float32:
+        return TG_F32
+    raise TypeError("logits must be bfloat16 or float32")
+
+
+def tree_attn(q, k_cache, v_cache, prefix_len, parent, node_off, max_nodes, *, scale=0.0,
+              out=None, lse_out=None, stream=None):
+    """Ancestor-masked GQA tree attention.  q [n_total, Hq, D] bf16,
+    k_cache / v_cache [B, Hkv, S_max, D] bf16, prefix_len [B] int32,
+    parent [n_total] int32 (local ids), node_off [B+1] int32.
+    Returns (out [n_total, Hq, D] bf16, lse_out or None)."""
+    _need(q, torch.bfloat16, "q")
+    _need(k_cache, torch.bfloat16, "k_cache")
+    _need(v_cache, torch.bfloat16, "v_cache")
+    for t, nm in ((prefix_len, "prefix_len"), (parent, "parent"), (node_off, "node_off")):
+        _need(t, torch.int32, nm)
+    n_total, Hq, D = q.shape
+    B, Hkv, S_max, D2 = k_cache.shape
+    if D2 != D or tuple(v_cache.shape) != tuple(k_cache.shape):
+        raise ValueError("q / k_cache / v_cache shapes disagree")
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, torch.bfloat16, "out")
+    if lse_out is not None:
+        _need(lse_out, torch.float32, "lse_out")
+    st = lib().treegraft_tree_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(prefix_len),
+                                   _ptr(parent), _ptr(node_off), B, int(max_nodes), n_total, Hq,
+                                   Hkv, D, S_max, float(scale), _ptr(out), _ptr(lse_out),
+                                   _stream(stream))
+    _check("treegraft_tree_attn", st)
+    return out, lse_out
+
+
+def expand_topk(logits, parent_score, k, *, row_idx=None, V=None, out=None, lse_out=None,
+                stream=None):
+    """Per-row log-softmax + exact top-k + cumulative score.  logits
+    [logit_rows, ld] bf16/fp32 (V <= ld columns used), parent_score [rows]
+    fp32, row_idx [rows] int32 or None.  Returns (tok, logprob, score, lse)."""
+    if logits.dim() != 2 or logits.stride(1) != 1:
+        raise ValueError("logits must be 2-D with unit column stride")
+    if not logits.is_cuda:
+        raise ValueError("logits must live on a CUDA device")
+    dt = _logit_dtype(logits)
+    _need(parent_score, torch.float32, "parent_score")
+    rows = parent_score.shape[0]
+    if row_idx is not None:
+        _need(row_idx, torch.int32, "row_idx")
+    V = logits.shape[1] if V is None else int(V)
+    dev = logits.device
+    if out is None:
+        out = (torch.empty(rows, k, dtype=torch.int32, device=dev),
+               torch.empty(rows, k, dtype=torch.float32, device=dev),
+               torch.empty(rows, k, dtype=torch.float32, device=dev))
+    tok, lp, sc = out
+    st = lib().treegraft_expand_topk(_ptr(logits), dt, logits.shape[0], V, logits.stride(0), rows,
+                                     _ptr(row_idx), _ptr(parent_score), int(k), _ptr(tok),
+                                     _ptr(lp), _ptr(sc), _ptr(lse_out), _stream(stream))
+    _check("treegraft_expand_topk", st)
+    return tok, lp, sc, lse_out
+
+
+def rescore_select(weak_edge, strong_lp, parent, token, visited, node_off, max_nodes, N, *,
+                   V=None, out=None, stream=None):
+    """Stronger-drafter rescoring + top-N reselection.  Returns (edge, score,
+    selected [B, N], n_selected [B])."""
+    _need(weak_edge, torch.float32, "weak_edge")
+    if strong_lp.dim() != 2 or strong_lp.stride(1) != 1 or strong_lp.dtype != torch.float32:
+        raise ValueError("strong_lp must be 2-D float32 with unit column stride")
+    for t, nm in ((parent, "parent"), (token, "token"), (node_off, "node_off")):
+        _need(t, torch.int32, nm)
+    _need(visited, torch.uint8, "visited")
+    n_total = parent.shape[0]
+    B = node_off.shape[0] - 1
+    V = strong_lp.shape[1] if V is None else int(V)
+    dev = parent.device
+    if out is None:
+        out = (torch.empty(n_total, dtype=torch.float32, device=dev),
+               torch.empty(n_total, dtype=torch.float32, device=dev),
+               torch.empty(B, N, dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev))
+    e, s, sel, nsel = out
+    st = lib().treegraft_rescore_select(_ptr(weak_edge), _ptr(strong_lp), V, strong_lp.stride(0),
+                                        _ptr(parent), _ptr(token), _ptr(visited), _ptr(node_off),
+                                        B, int(max_nodes), n_total, int(N), _ptr(e), _ptr(s),
+                                        _ptr(sel), _ptr(nsel), _stream(stream))
+    _check("treegraft_rescore_select", st)
+    return e, s, sel, nsel
+
+
+def accept_workspace_size(B: int, n_total: int) -> int:
+    return int(lib().treegraft_accept_workspace_size(B, n_total))
+
+
+def accept_workspace(B: int, n_total: int, device) -> torch.Tensor:
+    """A zero-filled workspace for accept (zeroed once; calls keep it ready)."""
+    nbytes = accept_workspace_size(B, n_total)
+    return torch.zeros(nbytes, dtype=torch.uint8, device=device)
+
+
+def accept(target_logits, token, parent, node_off, max_nodes, path_cap, ws, *, V=None,
+           out=None, stream=None):
+    """Greedy longest-accepted-path walk.  Returns (path [B, path_cap],
+    accept_len [B], bonus [B])."""
+    if target_logits.dim() != 2 or target_logits.stride(1) != 1 or not target_logits.is_cuda:
+        raise ValueError("target_logits must be a 2-D CUDA tensor with unit column stride")
+    dt = _logit_dtype(target_logits)
+    for t, nm in ((parent, "parent"), (token, "token"), (node_off, "node_off")):
+        _need(t, torch.int32, nm)
+    _need(ws, torch.uint8, "ws")
+    n_total = parent.shape[0]
+    B = node_off.shape[0] - 1
+    V = target_logits.shape[1] if V is None else int(V)
+    dev = parent.device
+    if out is None:
+        out = (torch.empty(B, path_cap, dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev))
+    path, alen, bonus = out
+    st = lib().treegraft_accept(_ptr(target_logits), dt, V, target_logits.stride(0), _ptr(token),
+                                _ptr(parent), _ptr(node_off), B, int(max_nodes), n_total,
+                                int(path_cap), _ptr(path), _ptr(alen), _ptr(bonus), _ptr(ws),
+                                ws.numel(), _stream(stream))
+    _check("treegraft_accept", st)
+    return path, alen, bonus
+
+
+def last_device_status(stream=None) -> int:
+    """Synchronise the stream; return and clear the device status bits."""
+    return int(lib().treegraft_last_device_status(_stream(stream)))

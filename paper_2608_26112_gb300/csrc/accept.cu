@@ -1,0 +1,200 @@
+// accept: greedy longest-accepted-path walk at temperature 0 (verification
+// step of Algorithms 1 and 2; greedy decoding setting of Appendix E).
+//
+// One launch.  Grid (C, n_total), clusters of C CTAs along x: each cluster
+// computes the target argmax (lowest token on ties) of one node row over
+// DSMEM, and its leader stores it in scratch and takes a ticket for the
+// row's tree.  The leader that draws the tree's last ticket performs the
+// walk for that tree with its 256 threads (one per node):
+//   ok[v]   = token[v] == am[pa(v)]
+//   full[v] = AND of ok over the root..v chain, depth[v] = its length
+//   a*      = argmax over full nodes of (depth, -id)
+// then writes the root..a* path, A = depth(a*) and the bonus token am[a*],
+// and resets the ticket so the scratch is ready for the next call.
+// Every node's row is scanned because the bonus token needs the row of a*,
+// which may be any node (a leaf included).
+#include <cooperative_groups.h>
+
+#include "launch.h"
+#include "rowscan.cuh"
+
+namespace cg = cooperative_groups;
+
+namespace tg {
+namespace {
+
+struct AcceptSmem {
+  uint64_t red[8];
+  uint64_t peer_key;
+  int tree, off, n, last;
+  int par[256];
+  int am[256];
+  uint32_t key[8];
+  int bad;
+};
+
+template <typename T, bool kAligned>
+__global__ void __launch_bounds__(kScanThreads) accept_kernel(AcceptArgs a, int row_base) {
+  __shared__ AcceptSmem sm;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int C = (int)cluster.num_blocks();
+  const int crank = (int)cluster.block_rank();
+  const int row = row_base + (int)blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int VW = ScanTraits<T>::kVW;
+  const int V = a.V;
+  const int per = ((V + C - 1) / C + VW - 1) / VW * VW;
+  const int c0 = min(V, crank * per);
+  const int c1 = min(V, c0 + per);
+  const T* rowp = reinterpret_cast<const T*>(a.logits) + (size_t)row * (size_t)a.ld;
+
+  uint4 buf[kScanVecs];
+  scan_load<T, kAligned>(rowp, c0, c1, buf);
+  float tmax;
+  int tpos;
+  scan_thread_max<T>(buf, c0, c1, tmax, tpos);
+  uint64_t key = (tpos < 0) ? 0ull : make_key(tmax, (uint32_t)tpos);
+  key = warp_max_u64(key);
+  if (lane == 0) sm.red[warp] = key;
+  __syncthreads();
+  if (tid == 0) {
+    uint64_t m = sm.red[0];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) m = sm.red[w] > m ? sm.red[w] : m;
+    sm.peer_key = m;
+  }
+  cluster.sync();
+  uint64_t best = 0;
+  if (crank == 0 && tid == 0) {
+    for (int c = 0; c < C; ++c) {
+      const uint64_t kc = cluster.map_shared_rank(&sm, c)->peer_key;
+      best = kc > best ? kc : best;
+    }
+  }
+  cluster.sync();
+  if (crank != 0) return;
+
+  // leader: publish the argmax, take a ticket for the row's tree
+  if (tid == 0) {
+    a.am[row] = (int32_t)key_index(best);
+    // tree of this row: last b with node_off[b] <= row
+    int lo = 0, hi = a.B - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.node_off[mid] <= row) lo = mid; else hi = mid - 1;
+    }
+    const int b = lo;
+    const int off = a.node_off[b];
+    const int n = a.node_off[b + 1] - off;
+    __threadfence();
+    const int t = atomicAdd(&a.tickets[b], 1);
+    sm.tree = b;
+    sm.off = off;
+    sm.n = n;
+    sm.last = (t == n - 1);
+    if (sm.last) {
+      __threadfence();
+      a.tickets[b] = 0;
+    }
+    sm.bad = (n < 1 || n > 256 || off < 0 || off + n > a.n_total) ? 1 : 0;
+    if (sm.bad) raise_status(a.status, kStTree);
+  }
+  __syncthreads();
+  if (!sm.last) return;
+
+  // ---- walk of tree b (this CTA saw every row of the tree finish)
+  const int b = sm.tree, off = sm.off, n = sm.n;
+  if (sm.bad) return;
+  int v_par = -1;
+  if (tid < n) {
+    v_par = a.parent[off + tid];
+    sm.par[tid] = v_par;
+    sm.am[tid] = __ldcg(&a.am[off + tid]);
+  }
+  const bool bad = (tid < n) && (tid == 0 ? (v_par != -1) : (v_par < 0 || v_par >= tid));
+  if (__syncthreads_or(bad)) {
+    if (tid == 0) raise_status(a.status, kStTree);
+    return;
+  }
+  uint32_t wkey = 0;
+  int depth = 0;
+  if (tid < n) {
+    bool full = true;
+    int v = tid;
+    while (v != 0) {  // parent[v] < v: at most v steps
+      const int p = sm.par[v];
+      full = full && (a.token[off + v] == sm.am[p]);
+      v = p;
+      ++depth;
+    }
+    wkey = full ? (((uint32_t)depth << 16) | (uint32_t)(0xFFFF - tid)) : 0u;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint32_t w = __shfl_xor_sync(0xffffffffu, wkey, o);
+    wkey = w > wkey ? w : wkey;
+  }
+  if (lane == 0) sm.key[warp] = wkey;
+  __syncthreads();
+  uint32_t best_w = sm.key[0];
+#pragma unroll
+  for (int w = 1; w < 8; ++w) best_w = sm.key[w] > best_w ? sm.key[w] : best_w;
+  const int A = (int)(best_w >> 16);
+  const int astar = 0xFFFF - (int)(best_w & 0xFFFF);
+  if (A + 1 > a.path_cap) {
+    if (tid == 0) raise_status(a.status, kStIndex);
+    return;
+  }
+  int32_t* path = a.path + (size_t)b * a.path_cap;
+  if (tid == 0) {
+    int v = astar;
+    for (int d = A; d >= 0; --d) {
+      path[d] = v;
+      v = sm.par[v];
+    }
+    a.accept_len[b] = A;
+    a.bonus[b] = sm.am[astar];
+  }
+  for (int d = A + 1 + tid; d < a.path_cap; d += kScanThreads) path[d] = -1;
+}
+
+template <typename T, bool kAligned>
+cudaError_t launch_accept_t(const AcceptArgs& a, int C, cudaStream_t s) {
+  auto kern = accept_kernel<T, kAligned>;
+  if (C > 8) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
+  for (int r0 = 0; r0 < a.n_total; r0 += 65535) {
+    const int nr = min(65535, a.n_total - r0);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(C, nr, 1);
+    cfg.blockDim = dim3(kScanThreads, 1, 1);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, a, r0);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s) {
+  const int C = scan_cluster_size(a.V, a.is_bf16, a.n_total, device_sm_count());
+  const int esz = a.is_bf16 ? 2 : 4;
+  const bool aligned = ((reinterpret_cast<uintptr_t>(a.logits) & 15) == 0) &&
+                       (((a.ld * esz) & 15) == 0);
+  if (a.is_bf16)
+    return aligned ? launch_accept_t<__nv_bfloat16, true>(a, C, s)
+                   : launch_accept_t<__nv_bfloat16, false>(a, C, s);
+  return aligned ? launch_accept_t<float, true>(a, C, s) : launch_accept_t<float, false>(a, C, s);
+}
+
+}  // namespace tg

@@ -1,0 +1,285 @@
+// C ABI of the library (declared in include/treegraft.h): host-side argument
+// validation, TMA descriptor encoding, the per-device status word, and the
+// calls into the kernel launchers.  Nothing here allocates device memory.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "../../include/treegraft.h"
+#include "launch.h"
+
+namespace tg {
+
+// One status word per device; kernels OR bits into it, the host reads and
+// clears it in treegraft_last_device_status().
+__device__ int g_status_word;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+int* g_status_ptr[kMaxDevices] = {};
+int g_sm_count[kMaxDevices] = {};
+
+int current_device() {
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= kMaxDevices) return -1;
+  return d;
+}
+
+int* status_ptr() {
+  const int d = current_device();
+  if (d < 0) return nullptr;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_status_ptr[d]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+    g_status_ptr[d] = static_cast<int*>(p);
+  }
+  return g_status_ptr[d];
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+bool encode_bf16(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims,
+                 const cuuint64_t* strides_bytes, const cuuint32_t* box) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), dims,
+            strides_bytes, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+}  // namespace
+
+int device_sm_count() {
+  const int d = current_device();
+  if (d < 0) return 148;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_sm_count[d]) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, d) != cudaSuccess || n <= 0)
+      n = 148;
+    g_sm_count[d] = n;
+  }
+  return g_sm_count[d];
+}
+
+}  // namespace tg
+
+using namespace tg;
+
+extern "C" {
+
+int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
+                        const int32_t* prefix_len, const int32_t* parent, const int32_t* node_off,
+                        int B, int max_nodes, int n_total, int Hq, int Hkv, int D, int S_max,
+                        float scale, void* out, float* lse_out, void* stream) {
+  if (!q || !k_cache || !v_cache || !prefix_len || !parent || !node_off || !out)
+    return TG_ERR_INVALID_ARG;
+  if (B < 1 || max_nodes < 1 || max_nodes > TG_MAX_TREE_NODES || n_total < 1 || Hq < 1 ||
+      Hkv < 1 || S_max < 1 || !(scale >= 0.f) || !std::isfinite(scale))
+    return TG_ERR_INVALID_ARG;
+  if (Hq % Hkv) return TG_ERR_INVALID_ARG;
+  if ((long long)n_total > (long long)B * max_nodes || max_nodes > S_max) return TG_ERR_INVALID_ARG;
+  const int G = Hq / Hkv;
+  if (D != 64 && D != 128) return TG_ERR_UNSUPPORTED;
+  if (G != 1 && G != 2 && G != 4 && G != 8) return TG_ERR_UNSUPPORTED;
+  if ((long long)B * Hkv > 65535 || (long long)B * Hkv * S_max + 128 >= (1ll << 31))
+    return TG_ERR_UNSUPPORTED;
+  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out))
+    return TG_ERR_INVALID_ARG;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+
+  CUtensorMap tq, tk, tv;
+  {
+    const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hq, (cuuint64_t)n_total};
+    const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hq * D * 2};
+    const cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(128 / G)};
+    if (!encode_bf16(&tq, q, 3, dims, strides, box)) return TG_ERR_CUDA;
+  }
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)B * Hkv * S_max};
+    const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+    const cuuint32_t box[2] = {64, 128};
+    if (!encode_bf16(&tk, k_cache, 2, dims, strides, box)) return TG_ERR_CUDA;
+    if (!encode_bf16(&tv, v_cache, 2, dims, strides, box)) return TG_ERR_CUDA;
+  }
+  AttnArgs a;
+  a.prefix_len = prefix_len;
+  a.parent = parent;
+  a.node_off = node_off;
+  a.B = B;
+  a.max_nodes = max_nodes;
+  a.n_total = n_total;
+  a.Hq = Hq;
+  a.Hkv = Hkv;
+  a.D = D;
+  a.S_max = S_max;
+  const float sc = scale > 0.f ? scale : 1.0f / std::sqrt((float)D);
+  a.scale_log2 = sc * 1.4426950408889634f;
+  a.out = out;
+  a.lse_out = lse_out;
+  a.status = st;
+  const int mtiles = (G * max_nodes + 127) / 128;
+  const int splits = tree_attn_pick_splits(B, Hkv, mtiles, S_max, device_sm_count());
+  return launch_tree_attn(tq, tk, tv, a, splits, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? TG_OK
+             : TG_ERR_CUDA;
+}
+
+int treegraft_expand_topk(const void* logits, int dtype, int logit_rows, int V, int64_t ld,
+                          int rows, const int32_t* row_idx, const float* parent_score, int k,
+                          int32_t* tok, float* logprob, float* score, float* lse_out,
+                          void* stream) {
+  if (rows == 0) return TG_OK;
+  if (!logits || !parent_score || !tok || !logprob || !score) return TG_ERR_INVALID_ARG;
+  if (dtype != TG_BF16 && dtype != TG_F32) return TG_ERR_INVALID_ARG;
+  if (rows < 0 || V < 1 || ld < V || logit_rows < 1 || k < 1 || k > V) return TG_ERR_INVALID_ARG;
+  if (!row_idx && logit_rows < rows) return TG_ERR_INVALID_ARG;
+  if (k > TG_MAX_TOPK || V > (dtype == TG_BF16 ? 262144 : 131072)) return TG_ERR_UNSUPPORTED;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  TopkArgs a;
+  a.logits = logits;
+  a.is_bf16 = dtype == TG_BF16;
+  a.logit_rows = logit_rows;
+  a.V = V;
+  a.ld = ld;
+  a.rows = rows;
+  a.row_idx = row_idx;
+  a.parent_score = parent_score;
+  a.k = k;
+  a.tok = tok;
+  a.logprob = logprob;
+  a.score = score;
+  a.lse_out = lse_out;
+  a.status = st;
+  return launch_expand_topk(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK
+                                                                               : TG_ERR_CUDA;
+}
+
+int treegraft_rescore_select(const float* weak_edge, const float* strong_lp, int V, int64_t ld,
+                             const int32_t* parent, const int32_t* token, const uint8_t* visited,
+                             const int32_t* node_off, int B, int max_nodes, int n_total, int N,
+                             float* edge_out, float* score_out, int32_t* selected,
+                             int32_t* n_selected, void* stream) {
+  if (!weak_edge || !strong_lp || !parent || !token || !visited || !node_off || !edge_out ||
+      !score_out || !selected || !n_selected)
+    return TG_ERR_INVALID_ARG;
+  if (B < 1 || V < 1 || ld < V || max_nodes < 1 || max_nodes > TG_MAX_TREE_NODES || N < 1 ||
+      N > TG_MAX_TREE_NODES || n_total < B || (long long)n_total > (long long)B * max_nodes)
+    return TG_ERR_INVALID_ARG;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  RescoreArgs a;
+  a.weak_edge = weak_edge;
+  a.strong_lp = strong_lp;
+  a.V = V;
+  a.ld = ld;
+  a.parent = parent;
+  a.token = token;
+  a.visited = visited;
+  a.node_off = node_off;
+  a.B = B;
+  a.N = N;
+  a.n_total = n_total;
+  a.edge_out = edge_out;
+  a.score_out = score_out;
+  a.selected = selected;
+  a.n_selected = n_selected;
+  a.status = st;
+  return launch_rescore_select(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK
+                                                                                  : TG_ERR_CUDA;
+}
+
+size_t treegraft_accept_workspace_size(int B, int n_total) {
+  if (B < 1 || n_total < 1) return 0;
+  const size_t bytes = ((size_t)n_total + (size_t)B) * sizeof(int32_t);
+  return (bytes + 255) & ~(size_t)255;
+}
+
+int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld, const int32_t* token,
+                     const int32_t* parent, const int32_t* node_off, int B, int max_nodes,
+                     int n_total, int path_cap, int32_t* path, int32_t* accept_len,
+                     int32_t* bonus, void* ws, size_t ws_bytes, void* stream) {
+  if (!target_logits || !token || !parent || !node_off || !path || !accept_len || !bonus || !ws)
+    return TG_ERR_INVALID_ARG;
+  if (dtype != TG_BF16 && dtype != TG_F32) return TG_ERR_INVALID_ARG;
+  if (B < 1 || V < 1 || ld < V || n_total < 1 || path_cap < 1 || max_nodes < 1 ||
+      max_nodes > TG_MAX_TREE_NODES || (long long)n_total > (long long)B * max_nodes)
+    return TG_ERR_INVALID_ARG;
+  if (ws_bytes < treegraft_accept_workspace_size(B, n_total) || !aligned16(ws))
+    return TG_ERR_INVALID_ARG;
+  if (V > (dtype == TG_BF16 ? 262144 : 131072)) return TG_ERR_UNSUPPORTED;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  AcceptArgs a;
+  a.logits = target_logits;
+  a.is_bf16 = dtype == TG_BF16;
+  a.V = V;
+  a.ld = ld;
+  a.token = token;
+  a.parent = parent;
+  a.node_off = node_off;
+  a.B = B;
+  a.n_total = n_total;
+  a.path_cap = path_cap;
+  a.path = path;
+  a.accept_len = accept_len;
+  a.bonus = bonus;
+  a.am = static_cast<int32_t*>(ws);
+  a.tickets = static_cast<int32_t*>(ws) + n_total;
+  a.status = st;
+  return launch_accept(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK : TG_ERR_CUDA;
+}
+
+int treegraft_last_device_status(void* stream) {
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return TG_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, st, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return TG_ERR_CUDA;
+  if (v != 0 && cudaMemset(st, 0, sizeof(int)) != cudaSuccess) return TG_ERR_CUDA;
+  return v;
+}
+
+const char* treegraft_status_string(int status) {
+  switch (status) {
+    case TG_OK: return "ok";
+    case TG_ERR_INVALID_ARG: return "invalid argument";
+    case TG_ERR_UNSUPPORTED: return "unsupported configuration";
+    case TG_ERR_CUDA: return "CUDA error";
+    case TG_ERR_DEVICE_TREE: return "malformed tree seen on the device";
+    case TG_ERR_TIMEOUT: return "bounded device wait gave up";
+    case TG_ERR_DEVICE_INDEX: return "index out of range seen on the device";
+    default: return "combination of device status bits";
+  }
+}
+
+}  // extern "C"

@@ -1,0 +1,83 @@
+// Internal launchers (host side) called by the C ABI layer in api.cu.  All
+// arguments are validated by the caller; these only size grids and launch.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace tg {
+
+struct AttnArgs {
+  const int32_t* prefix_len;
+  const int32_t* parent;
+  const int32_t* node_off;
+  int B, max_nodes, n_total, Hq, Hkv, D, S_max;
+  float scale_log2;  // softmax scale * log2(e)
+  void* out;
+  float* lse_out;
+  int* status;
+};
+// tmaps: q [D, Hq, n_total], k and v [D, B*Hkv*S_max] (innermost first)
+cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
+                             const CUtensorMap& tm_v, const AttnArgs& a, int kv_splits,
+                             cudaStream_t s);
+int tree_attn_pick_splits(int B, int Hkv, int mtiles, int S_max, int num_sms);
+
+struct TopkArgs {
+  const void* logits;
+  int is_bf16;
+  int logit_rows, V;
+  int64_t ld;
+  int rows;
+  const int32_t* row_idx;
+  const float* parent_score;
+  int k;
+  int32_t* tok;
+  float* logprob;
+  float* score;
+  float* lse_out;
+  int* status;
+};
+cudaError_t launch_expand_topk(const TopkArgs& a, cudaStream_t s);
+int scan_cluster_size(int V, int is_bf16, int rows, int num_sms);
+
+struct RescoreArgs {
+  const float* weak_edge;
+  const float* strong_lp;
+  int V;
+  int64_t ld;
+  const int32_t* parent;
+  const int32_t* token;
+  const uint8_t* visited;
+  const int32_t* node_off;
+  int B, N, n_total;
+  float* edge_out;
+  float* score_out;
+  int32_t* selected;
+  int32_t* n_selected;
+  int* status;
+};
+cudaError_t launch_rescore_select(const RescoreArgs& a, cudaStream_t s);
+
+struct AcceptArgs {
+  const void* logits;
+  int is_bf16;
+  int V;
+  int64_t ld;
+  const int32_t* token;
+  const int32_t* parent;
+  const int32_t* node_off;
+  int B, n_total, path_cap;
+  int32_t* path;
+  int32_t* accept_len;
+  int32_t* bonus;
+  int32_t* am;       // scratch [n_total]
+  int32_t* tickets;  // scratch [B], zero between calls
+  int* status;
+};
+cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s);
+
+int device_sm_count();
+
+}  // namespace tg

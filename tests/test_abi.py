@@ -1,0 +1,120 @@
+"""The C-ABI library builds, loads and exports every entry point that
+include/treegraft.h declares; host-side argument validation rejects bad
+calls before anything reaches the GPU.  CPU only: no kernel is launched."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "treegraft.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(treegraft_\w+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_26112_gb300 import build
+    build.build()
+    from paper_2608_26112_gb300 import binding
+    return binding.lib()
+
+
+def test_header_declares_the_four_calls():
+    fns = declared_functions()
+    for name in ("treegraft_tree_attn", "treegraft_expand_topk", "treegraft_rescore_select",
+                 "treegraft_accept"):
+        assert name in fns
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    assert lib.treegraft_status_string(0) == b"ok"
+    assert b"invalid" in lib.treegraft_status_string(1)
+
+
+def test_workspace_size(lib):
+    assert lib.treegraft_accept_workspace_size(1, 60) >= 61 * 4
+    assert lib.treegraft_accept_workspace_size(1, 60) % 256 == 0
+    assert lib.treegraft_accept_workspace_size(0, 60) == 0
+
+
+NULL = None
+
+
+def test_tree_attn_rejects_bad_args_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    # null pointer
+    assert lib.treegraft_tree_attn(NULL, fake, fake, fake, fake, fake, 1, 16, 16, 8, 8, 64, 144,
+                                   0.0, fake, NULL, NULL) == 1
+    # head_dim 96 unsupported, G = 3 unsupported, Hq % Hkv != 0 invalid
+    assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 16, 16, 8, 8, 96, 144,
+                                   0.0, fake, NULL, NULL) == 2
+    assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 16, 16, 12, 4, 64, 144,
+                                   0.0, fake, NULL, NULL) == 2
+    assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 16, 16, 8, 3, 64, 144,
+                                   0.0, fake, NULL, NULL) == 1
+    # more than 256 nodes per tree
+    assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 300, 300, 8, 8, 64,
+                                   400, 0.0, fake, NULL, NULL) == 1
+    # misaligned q
+    assert lib.treegraft_tree_attn(ctypes.c_void_p(0x1002), fake, fake, fake, fake, fake, 1, 16,
+                                   16, 8, 8, 64, 144, 0.0, fake, NULL, NULL) == 1
+    # negative scale
+    assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 16, 16, 8, 8, 64, 144,
+                                   -1.0, fake, NULL, NULL) == 1
+
+
+def test_expand_topk_rejects_bad_args_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    args = dict(logits=fake, dtype=0, logit_rows=4, V=100, ld=100, rows=4, row_idx=NULL,
+                ps=fake, k=4)
+
+    def call(**kw):
+        a = dict(args, **kw)
+        return lib.treegraft_expand_topk(a["logits"], a["dtype"], a["logit_rows"], a["V"],
+                                         a["ld"], a["rows"], a["row_idx"], a["ps"], a["k"], fake,
+                                         fake, fake, NULL, NULL)
+    assert call(rows=0) == 0                 # empty call is a no-op
+    assert call(logits=NULL) == 1
+    assert call(k=101) == 1                  # k > V
+    assert call(k=0) == 1
+    assert call(k=33) == 2                   # beyond the top-k limit
+    assert call(ld=50) == 1                  # ld < V
+    assert call(dtype=7) == 1
+    assert call(rows=5) == 1                 # more rows than logits, no row_idx
+    assert call(V=300000, ld=300000) == 2
+
+
+def test_rescore_and_accept_reject_bad_args_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    assert lib.treegraft_rescore_select(fake, fake, 100, 100, fake, fake, fake, fake, 1, 64, 64,
+                                        0, fake, fake, fake, fake, NULL) == 1      # N = 0
+    assert lib.treegraft_rescore_select(fake, fake, 100, 100, fake, fake, fake, fake, 1, 300, 64,
+                                        8, fake, fake, fake, fake, NULL) == 1      # max_nodes
+    assert lib.treegraft_rescore_select(NULL, fake, 100, 100, fake, fake, fake, fake, 1, 64, 64,
+                                        8, fake, fake, fake, fake, NULL) == 1
+    ws = lib.treegraft_accept_workspace_size(1, 60)
+    assert lib.treegraft_accept(fake, 0, 100, 100, fake, fake, fake, 1, 60, 60, 8, fake, fake,
+                                fake, fake, ws - 1, NULL) == 1                     # ws too small
+    assert lib.treegraft_accept(fake, 0, 100, 100, fake, fake, fake, 1, 60, 60, 0, fake, fake,
+                                fake, fake, ws, NULL) == 1                         # path_cap 0
+    assert lib.treegraft_accept(fake, 0, 100, 100, fake, fake, fake, 1, 60, 61, 8, fake, fake,
+                                fake, fake, ws, NULL) == 1                         # n_total > B*max
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    from paper_2608_26112_gb300 import binding
+    monkeypatch.setattr(binding, "_lib", None)
+    monkeypatch.setattr(binding, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        binding.lib()

@@ -1,0 +1,352 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle on seeded
+synthetic inputs.  Bars: top-k indices, reselected sets and accepted paths
+bit-exact (ties to the lower token / node id); attention max-abs 2e-2 and
+mean-abs 2e-3 on bf16 outputs; path scores 1e-4 relative."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2608_26112_gb300 as tg
+from oracle import treegraft_oracle as O
+from paper_2608_26112_gb300 import synth
+from tests import _dev
+
+pytestmark = pytest.mark.gpu
+
+ATT_MAX_ABS, ATT_MEAN_ABS, LSE_ABS = 2e-2, 2e-3, 2e-3
+SCORE_RTOL = 1e-4
+
+
+@pytest.fixture(scope="module")
+def dev():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_26112_gb300 import build
+    build.build()
+    return torch.device("cuda:0")
+
+
+def _status_clean():
+    assert tg.last_device_status() == 0
+
+
+# ------------------------------------------------------------------ tree attention
+
+def _attn_shape(B, P, n, depth, Hq, Hkv, D, cap=None):
+    return dict(B=B, P=P, n=n, depth=depth, cap=cap, rank_bias=0.3, Hq=Hq, Hkv=Hkv, D=D, V=64,
+                logit_dtype="f32", k=4, N=4)
+
+
+ATTN_CASES = {
+    "tiny": "tiny",
+    "graft-mha": "graft-mha",
+    "llama3-8b-verify": "llama3-8b-verify",
+    "g1-d64-p1-n2": _attn_shape(1, 1, 2, 1, 4, 4, 64),
+    "g2-d128-p127-n33": _attn_shape(1, 127, 33, 5, 8, 4, 128),
+    "g8-d128-p129-n255": _attn_shape(1, 129, 255, 9, 64, 8, 128, cap=16),
+    "g4-d64-p0-n256": _attn_shape(1, 0, 256, 8, 16, 4, 64),
+    "g4-d128-n1": _attn_shape(2, [300, 17], [1, 1], 1, 32, 8, 128),
+    "ragged-b3": _attn_shape(3, [5, 300, 1000], [2, 64, 128], [1, 6, 8], 32, 8, 128, cap=10),
+    "n31-n32": _attn_shape(2, [128, 256], [31, 32], [3, 4], 16, 8, 64),
+    "g8-d64-b2": _attn_shape(2, [64, 200], [40, 50], [5, 6], 64, 8, 64, cap=10),
+}
+
+
+def _run_attn(wl, dev):
+    sh = wl["shape"]
+    q = _dev.bf16(wl["q"], dev)
+    k = _dev.bf16(wl["k_cache"], dev)
+    v = _dev.bf16(wl["v_cache"], dev)
+    lse = torch.full((q.shape[0], q.shape[1]), float("nan"), device=dev)
+    out, _ = tg.tree_attn(q, k, v, _dev.i32(wl["prefix_len"], dev), _dev.i32(wl["parent"], dev),
+                          _dev.i32(wl["node_off"], dev), _dev.max_nodes(wl), lse_out=lse)
+    _status_clean()
+    return _dev.bf16_to_np(out), lse.cpu().numpy().astype(np.float64)
+
+
+def _check_attn(wl, o, lse, oracle_o, oracle_lse):
+    err = np.abs(o - oracle_o)
+    assert np.isfinite(o).all()
+    assert err.max() <= ATT_MAX_ABS, err.max()
+    assert err.mean() <= ATT_MEAN_ABS, err.mean()
+    np.testing.assert_allclose(lse, oracle_lse, atol=LSE_ABS, rtol=0)
+
+
+@pytest.mark.parametrize("case", list(ATTN_CASES))
+def test_tree_attn_matches_oracle(dev, case):
+    wl = synth.make_workload(ATTN_CASES[case], seed=1, with_logits=False, with_strong=False)
+    o, lse = _run_attn(wl, dev)
+    ref_o, ref_lse = O.tree_attention(wl["q"], wl["k_cache"], wl["v_cache"], wl["prefix_len"],
+                                      wl["parent"], wl["node_off"], Hkv=wl["shape"]["Hkv"])
+    _check_attn(wl, o, lse, ref_o, ref_lse)
+
+
+def test_tree_attn_ignores_nan_past_the_sequence(dev):
+    wl = synth.make_workload(_attn_shape(2, [100, 61], [20, 67], [3, 5], 16, 4, 128), seed=2,
+                             kv_tail="nan", with_logits=False, with_strong=False, S_max=300)
+    o, lse = _run_attn(wl, dev)
+    ref_o, ref_lse = O.tree_attention(wl["q"], wl["k_cache"], wl["v_cache"], wl["prefix_len"],
+                                      wl["parent"], wl["node_off"], Hkv=4)
+    _check_attn(wl, o, lse, ref_o, ref_lse)
+
+
+def test_tree_attn_chain_equals_causal(dev):
+    # chain tree: the kernel's result must equal causal attention (oracle pin)
+    shape = _attn_shape(1, 200, 40, 39, 32, 8, 128)
+    wl = synth.make_workload(shape, seed=3, with_logits=False, with_strong=False)
+    wl["parent"] = np.arange(-1, 39, dtype=np.int32)
+    o, lse = _run_attn(wl, dev)
+    ref_o, ref_lse = O.tree_attention(wl["q"], wl["k_cache"], wl["v_cache"], wl["prefix_len"],
+                                      wl["parent"], wl["node_off"], Hkv=8)
+    _check_attn(wl, o, lse, ref_o, ref_lse)
+
+
+def test_tree_attn_llama70b_shape_sampled(dev):
+    # full 4 x (8192 + 128) Llama-3-70B-shaped launch; oracle on trees 0 and 3
+    wl = synth.make_workload("llama3-70b-verify", seed=0, with_logits=False, with_strong=False)
+    o, lse = _run_attn(wl, dev)
+    off = wl["node_off"]
+    for b in (0, 3):
+        a, e = int(off[b]), int(off[b + 1])
+        ref_o, ref_lse = O.tree_attention(wl["q"][a:e], wl["k_cache"][b:b + 1],
+                                          wl["v_cache"][b:b + 1], wl["prefix_len"][b:b + 1],
+                                          wl["parent"][a:e], [0, e - a], Hkv=8)
+        _check_attn(wl, o[a:e], lse[a:e], ref_o, ref_lse)
+
+
+def test_tree_attn_malformed_tree_sets_status(dev):
+    wl = synth.make_workload(_attn_shape(1, 16, 8, 3, 8, 8, 64), seed=4, with_logits=False,
+                             with_strong=False)
+    bad = wl["parent"].copy()
+    bad[5] = 6                                           # parent after child
+    q = _dev.bf16(wl["q"], dev)
+    out = torch.zeros_like(q)
+    tg.tree_attn(q, _dev.bf16(wl["k_cache"], dev), _dev.bf16(wl["v_cache"], dev),
+                 _dev.i32(wl["prefix_len"], dev), _dev.i32(bad, dev),
+                 _dev.i32(wl["node_off"], dev), 8, out=out)
+    assert tg.last_device_status() & 4
+    assert tg.last_device_status() == 0                  # cleared by the read
+
+
+# ------------------------------------------------------------------ expand_topk
+
+def _run_expand(lg_dev, ps, k, dev, row_idx=None, V=None):
+    rows = len(ps)
+    lse = torch.empty(rows, device=dev)
+    tok, lp, sc, _ = tg.expand_topk(lg_dev, _dev.f32(ps, dev), k,
+                                    row_idx=None if row_idx is None else _dev.i32(row_idx, dev),
+                                    V=V, lse_out=lse)
+    _status_clean()
+    return tok.cpu().numpy(), lp.cpu().numpy(), sc.cpu().numpy(), lse.cpu().numpy()
+
+
+def _check_expand(got, ref):
+    tok, lp, sc, lse = got
+    rtok, rlp, rsc, rlse = ref
+    np.testing.assert_array_equal(tok, rtok)
+    np.testing.assert_allclose(lp, rlp, rtol=SCORE_RTOL, atol=1e-5)
+    np.testing.assert_allclose(sc, rsc, rtol=SCORE_RTOL, atol=1e-5)
+    np.testing.assert_allclose(lse, rlse, rtol=1e-5, atol=1e-5)
+
+
+@pytest.mark.parametrize("name", ["tiny", "llama3-8b-verify", "graft-mha"])
+def test_expand_topk_workloads(dev, name):
+    wl = synth.make_workload(name, seed=0, with_strong=False)
+    bf = wl["logits"].dtype == np.uint16
+    k = wl["shape"]["k"]
+    got = _run_expand(_dev.logits(wl, dev), wl["parent_score"], k, dev)
+    ref = O.expand_topk(wl["logits"], wl["parent_score"], k, bf16=bf)
+    _check_expand(got, ref)
+
+
+@pytest.mark.parametrize("V,ld,dtype,k", [(1023, 1024, "f32", 5), (32001, 32001, "bf16", 10),
+                                          (32001, 32008, "bf16", 32), (777, 801, "f32", 1),
+                                          (100, 100, "bf16", 32), (262144, 262144, "bf16", 16)])
+def test_expand_topk_ragged_vocab(dev, V, ld, dtype, k):
+    rng = synth.make_rng(V + k)
+    rows = 7
+    x = synth.normal_f32(rng, (rows, ld), 3.0)
+    ps = synth.normal_f32(rng, (rows,), 2.0)
+    if dtype == "bf16":
+        bits = synth.f32_to_bf16_bits(x)
+        got = _run_expand(_dev.bf16(bits, dev), ps, k, dev, V=V)
+        ref = O.expand_topk(bits[:, :V], ps, k, bf16=True)
+    else:
+        got = _run_expand(_dev.f32(x, dev), ps, k, dev, V=V)
+        ref = O.expand_topk(x[:, :V], ps, k)
+    _check_expand(got, ref)
+
+
+def test_expand_topk_ties_inf_and_row_idx(dev):
+    rng = synth.make_rng(5)
+    V = 5000
+    x = rng.integers(-1, 2, size=(6, V)).astype(np.float32)     # heavy ties
+    x[2] = -np.inf                                              # all -inf row
+    x[3, ::3] = -np.inf
+    x[4] = 0.0
+    x[4, 4999] = 0.5
+    x[5, :] = -0.0
+    x[5, 17] = 0.0
+    ps = np.array([0, -1, -2, -3, -4, -5, -6, -7], np.float32)
+    row_idx = np.array([5, 4, 3, 0, 1, 0, 2, 2], np.int32)
+    got = _run_expand(_dev.f32(x, dev), ps, 12, dev, row_idx=row_idx)
+    ref = O.expand_topk(x, ps, 12, row_idx=row_idx)
+    np.testing.assert_array_equal(got[0], ref[0])
+    for g, r in zip(got[1:], ref[1:]):
+        np.testing.assert_array_equal(np.isneginf(g), np.isneginf(r))
+        fin = np.isfinite(r)
+        np.testing.assert_allclose(g[fin], r[fin], rtol=1e-5, atol=1e-5)
+
+
+def test_expand_topk_bad_row_idx_sets_status(dev):
+    x = torch.zeros(4, 64, device=dev)
+    tg.expand_topk(x, torch.zeros(2, device=dev), 3, row_idx=_dev.i32([1, 9], dev))
+    assert tg.last_device_status() & 16
+
+
+# ------------------------------------------------------------------ rescore_select
+
+def _run_rescore(wl, N, dev, visited=None):
+    vis = wl["visited"] if visited is None else visited
+    e, s, sel, ns = tg.rescore_select(_dev.f32(wl["weak_edge"], dev), _dev.f32(wl["strong_lp"], dev),
+                                      _dev.i32(wl["parent"], dev), _dev.i32(wl["token"], dev),
+                                      _dev.u8(vis, dev), _dev.i32(wl["node_off"], dev),
+                                      _dev.max_nodes(wl), N)
+    _status_clean()
+    return e.cpu().numpy(), s.cpu().numpy(), sel.cpu().numpy(), ns.cpu().numpy()
+
+
+@pytest.mark.parametrize("name,visited", [("tiny", None), ("llama3-8b-verify", None),
+                                          ("graft-mha", "none"), ("graft-mha", "all"),
+                                          ("llama3-70b-verify", None)])
+def test_rescore_select_bit_exact(dev, name, visited):
+    wl = synth.make_workload(name, seed=0, with_logits=False)
+    vis = {None: wl["visited"], "none": np.zeros_like(wl["visited"]),
+           "all": np.ones_like(wl["visited"])}[visited]
+    N = wl["shape"]["N"]
+    got = _run_rescore(wl, N, dev, vis)
+    ref = O.rescore_select(wl["weak_edge"], wl["strong_lp"], wl["parent"], wl["token"], vis,
+                           wl["node_off"], N)
+    for g, r in zip(got, ref):
+        np.testing.assert_array_equal(g, r)
+
+
+# ------------------------------------------------------------------ accept
+
+def _run_accept(wl, dev, path_cap, lg=None):
+    B = len(wl["node_off"]) - 1
+    ws = tg.accept_workspace(B, len(wl["parent"]), dev)
+    lg = _dev.logits(wl, dev) if lg is None else lg
+    path, alen, bonus = tg.accept(lg, _dev.i32(wl["token"], dev), _dev.i32(wl["parent"], dev),
+                                  _dev.i32(wl["node_off"], dev), _dev.max_nodes(wl), path_cap, ws)
+    _status_clean()
+    return path.cpu().numpy(), alen.cpu().numpy(), bonus.cpu().numpy(), ws
+
+
+@pytest.mark.parametrize("name,bump", [("tiny", 8.0), ("tiny", 40.0), ("llama3-8b-verify", 8.0),
+                                       ("llama3-8b-verify", 40.0), ("llama3-70b-verify", 40.0),
+                                       ("graft-mha", 40.0)])
+def test_accept_bit_exact(dev, name, bump):
+    wl = synth.make_workload(name, seed=7, with_strong=False)
+    if bump != 8.0:
+        # re-plant with a larger bump so that long accepted paths occur
+        wl = synth.make_workload(name, seed=7, with_strong=False, with_logits=False)
+        rng = synth.make_rng(99)
+        lg = synth.normal_f32(rng, (len(wl["parent"]), wl["shape"]["V"]), 3.0)
+        off = wl["node_off"]
+        for b in range(len(off) - 1):
+            a, e = int(off[b]), int(off[b + 1])
+            synth.plant_child_bump(rng, lg, wl["parent"][a:e], wl["token"][a:e], np.arange(a, e),
+                                   prob=0.9, bump=bump)
+        wl["logits"] = lg if wl["shape"]["logit_dtype"] == "f32" else synth.f32_to_bf16_bits(lg)
+    bf = wl["logits"].dtype == np.uint16
+    cap = _dev.max_nodes(wl)
+    got = _run_accept(wl, dev, cap)
+    ref = O.accept(wl["logits"], wl["token"], wl["parent"], wl["node_off"], cap, bf16=bf)
+    for g, r in zip(got[:3], ref):
+        np.testing.assert_array_equal(g, r)
+    if bump == 40.0:
+        assert ref[1].max() >= 1        # a planted child was accepted
+    # the workspace is ready for a second call: same answer
+    got2 = _run_accept(wl, dev, cap)
+    for g, r in zip(got2[:3], ref):
+        np.testing.assert_array_equal(g, r)
+
+
+def test_accept_path_cap_too_small_sets_status(dev):
+    n, V = 6, 50
+    parent = np.arange(-1, n - 1, dtype=np.int32)
+    token = np.arange(n, dtype=np.int32) + 3
+    x = np.zeros((n, V), np.float32)
+    for v in range(n - 1):
+        x[v, token[v + 1]] = 5.0
+    wl = dict(parent=parent, token=token, node_off=np.array([0, n], np.int32), logits=x)
+    ws = tg.accept_workspace(1, n, dev)
+    tg.accept(_dev.f32(x, dev), _dev.i32(token, dev), _dev.i32(parent, dev),
+              _dev.i32(wl["node_off"], dev), n, 3, ws)
+    assert tg.last_device_status() & 16
+    path, A, bonus, _ = _run_accept(wl, dev, n)
+    assert A[0] == n - 1 and list(path[0]) == list(range(n))
+
+
+def test_accept_grafting_examples(dev):
+    import json, os
+    with open(os.path.join(os.path.dirname(__file__), "golden", "grafting_examples.json")) as f:
+        cases = json.load(f)["cases"]
+    for case in cases:
+        parent = np.array(case["parent"], np.int32)
+        n, V = len(parent), case["vocab"]
+        x = np.zeros((n, V), np.float32)
+        x[np.arange(n), case["target_argmax"]] = 3.0
+        wl = dict(parent=parent, token=np.array(case["token"], np.int32),
+                  node_off=np.array([0, n], np.int32), logits=x)
+        path, A, bonus, _ = _run_accept(wl, dev, n)
+        exp = case["accepted_path"]
+        assert list(path[0, :len(exp)]) == exp and A[0] == len(exp) - 1
+        assert bonus[0] == case["bonus"]
+
+
+# ------------------------------------------------------------------ graft step pipeline
+
+def test_graft_step_pipeline(dev):
+    """Two-drafter grafting step: rescore all 64 weak-tree nodes, reselect 16
+    grafting positions, expand each by top-8 from the stronger drafter's
+    rows, graft the 128 children non-destructively (append), accept on the
+    192-node tree.  Every stage gets identical inputs on both sides."""
+    wl = synth.make_workload("graft-mha", seed=0, with_logits=False, with_strong=False)
+    rng = synth.make_rng(123)
+    n, V, N, k = 64, 32000, 16, 8
+    weak_lp = synth.normal_f32(rng, (n, V), 3.0, -np.log(V) - 4.5)
+    strong_lp = (weak_lp + synth.normal_f32(rng, (n, V), 0.5)).astype(np.float32)
+    weak_edge = np.zeros(n, np.float32)
+    for v in range(1, n):
+        weak_edge[v] = weak_lp[wl["parent"][v], wl["token"][v]]
+    visited = np.zeros(n, np.uint8)
+    # stage 1: rescore + reselect
+    e_g, s_g, sel_g, ns_g = tg.rescore_select(
+        _dev.f32(weak_edge, dev), _dev.f32(strong_lp, dev), _dev.i32(wl["parent"], dev),
+        _dev.i32(wl["token"], dev), _dev.u8(visited, dev), _dev.i32(wl["node_off"], dev), n, N)
+    e_o, s_o, sel_o, ns_o = O.rescore_select(weak_edge, strong_lp, wl["parent"], wl["token"],
+                                             visited, wl["node_off"], N)
+    np.testing.assert_array_equal(sel_g.cpu().numpy(), sel_o)
+    np.testing.assert_array_equal(s_g.cpu().numpy(), s_o)
+    sel = sel_o[0]
+    # stage 2: expand the selected nodes from the stronger drafter's rows
+    tok_g, lp_g, sc_g, _ = tg.expand_topk(_dev.f32(strong_lp, dev), s_g[torch.from_numpy(sel).long().to(dev)].contiguous(), k,
+                                          row_idx=_dev.i32(sel, dev))
+    tok_o, lp_o, sc_o, _ = O.expand_topk(strong_lp, s_o[sel], k, row_idx=sel)
+    np.testing.assert_array_equal(tok_g.cpu().numpy(), tok_o)
+    np.testing.assert_allclose(sc_g.cpu().numpy(), sc_o, rtol=SCORE_RTOL, atol=1e-5)
+    # stage 3: non-destructive graft (append children), then accept
+    parent = np.concatenate([wl["parent"], np.repeat(sel, k)]).astype(np.int32)
+    token = np.concatenate([wl["token"], tok_o.reshape(-1)]).astype(np.int32)
+    n2 = len(parent)
+    assert n2 == 192
+    tl = synth.normal_f32(rng, (n2, V), 3.0)
+    synth.plant_child_bump(rng, tl, parent, token, np.arange(n2), prob=0.9, bump=40.0)
+    tl_bits = synth.f32_to_bf16_bits(tl)
+    g = dict(parent=parent, token=token, node_off=np.array([0, n2], np.int32), logits=tl_bits)
+    path, A, bonus, _ = _run_accept(g, dev, n2)
+    rp, rA, rb = O.accept(tl_bits, token, parent, g["node_off"], n2, bf16=True)
+    np.testing.assert_array_equal(path, rp)
+    assert A[0] == rA[0] and bonus[0] == rb[0]
