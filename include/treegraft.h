@@ -190,6 +190,37 @@ int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld,
                      void* stream);
 
 /*
+ * treegraft_accept_noalloc - treegraft_accept for callers that cannot
+ * allocate device memory.
+ *
+ * The paper has no counterpart: this is a library convenience.  Some callers
+ * cannot obtain a scratch buffer - a plugin that an inference engine hands
+ * only its inputs and outputs, or code running where every device
+ * allocation must go through a pool it cannot reach.  This variant takes no
+ * `ws` and allocates nothing: its scratch lives in a fixed array inside the
+ * library, so every GPU that loads the library holds about 272 KB for it
+ * until the process exits.
+ *
+ * Arguments, outputs and results are those of treegraft_accept (without ws
+ * and ws_bytes).  Limits of the fixed array: n_total <= TG_NOALLOC_MAX_NODES
+ * and B <= TG_NOALLOC_MAX_TREES; larger calls return TG_ERR_UNSUPPORTED and
+ * launch nothing.
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * All calls on a device share the one array: calls that overlap on the GPU
+ * (other streams, other host threads) race and give wrong results; order
+ * them on one stream.  Each call clears the counters it needs on `stream`
+ * (cudaMemsetAsync) before its kernel runs.
+ */
+#define TG_NOALLOC_MAX_NODES 65536
+#define TG_NOALLOC_MAX_TREES 4096
+int treegraft_accept_noalloc(const void* target_logits, int dtype, int V, int64_t ld,
+                             const int32_t* token, const int32_t* parent,
+                             const int32_t* node_off, int B, int max_nodes, int n_total,
+                             int path_cap, int32_t* path, int32_t* accept_len, int32_t* bonus,
+                             void* stream);
+
+/*
  * treegraft_last_device_status - synchronise `stream`, return the OR of the
  * device status bits raised since the last call on the current device
  * (TG_OK if none), and clear them.  Returns TG_ERR_CUDA if the

@@ -45,6 +45,8 @@ _SIGNATURES = {
     "treegraft_accept_workspace_size": [_c_int, _c_int],
     "treegraft_accept": [_c_vp, _c_int, _c_int, _c_i64, _c_vp, _c_vp, _c_vp, _c_int, _c_int,
                          _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_size, _c_vp],
+    "treegraft_accept_noalloc": [_c_vp, _c_int, _c_int, _c_i64, _c_vp, _c_vp, _c_vp, _c_int,
+                                 _c_int, _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp],
     "treegraft_last_device_status": [_c_vp],
     "treegraft_status_string": [_c_int],
 }
@@ -221,6 +223,30 @@ def accept(target_logits, token, parent, node_off, max_nodes, path_cap, ws, *, V
                                 int(path_cap), _ptr(path), _ptr(alen), _ptr(bonus), _ptr(ws),
                                 ws.numel(), _stream(stream))
     _check("treegraft_accept", st)
+    return path, alen, bonus
+
+
+def accept_noalloc(target_logits, token, parent, node_off, max_nodes, path_cap, *, V=None,
+                   out=None, stream=None):
+    """accept() without a workspace, for callers that cannot allocate device
+    memory: the library keeps the scratch in a fixed per-device array
+    (n_total <= 65536, B <= 4096).  Calls that overlap on the GPU race."""
+    if target_logits.dim() != 2 or target_logits.stride(1) != 1 or not target_logits.is_cuda:
+        raise ValueError("target_logits must be a 2-D CUDA tensor with unit column stride")
+    dt = _logit_dtype(target_logits)
+    for t, nm in ((parent, "parent"), (token, "token"), (node_off, "node_off")):
+        _need(t, torch.int32, nm)
+    n_total = parent.shape[0]
+    B = node_off.shape[0] - 1
+    V = target_logits.shape[1] if V is None else int(V)
+    if out is None:
+        raise ValueError("accept_noalloc writes into caller-provided outputs: pass out=")
+    path, alen, bonus = out
+    st = lib().treegraft_accept_noalloc(_ptr(target_logits), dt, V, target_logits.stride(0),
+                                        _ptr(token), _ptr(parent), _ptr(node_off), B,
+                                        int(max_nodes), n_total, int(path_cap), _ptr(path),
+                                        _ptr(alen), _ptr(bonus), _stream(stream))
+    _check("treegraft_accept_noalloc", st)
     return path, alen, bonus
 
 

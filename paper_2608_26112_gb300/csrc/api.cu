@@ -88,6 +88,8 @@ int device_sm_count() {
   return g_sm_count[d];
 }
 
+int* status_word_ptr() { return status_ptr(); }
+
 }  // namespace tg
 
 using namespace tg;

@@ -79,5 +79,7 @@ struct AcceptArgs {
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s);
 
 int device_sm_count();
+// device address of the per-device status word (nullptr on failure)
+int* status_word_ptr();
 
 }  // namespace tg
