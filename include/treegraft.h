@@ -20,7 +20,8 @@
  *    rows [node_off[b], node_off[b+1]); inside a tree, parent[] holds LOCAL
  *    ids with parent[0] = -1 and 0 <= parent[i] < i (parents before
  *    children, the order Algorithm 3 re-indexes the verification tree into).
- *    Every tree has at least one node (its root) and at most 256 nodes.
+ *    node_off[0] = 0.  Every tree has at least one node (its root) and at
+ *    most 256 nodes.
  *  - bf16 data is IEEE bfloat16 (raw 16-bit patterns); all fp32/int32 data
  *    is native-endian.
  */
@@ -77,7 +78,8 @@ typedef enum { TG_BF16 = 0, TG_F32 = 1 } tg_dtype;
  * out      bf16 [n_total, Hq, D];  lse_out fp32 [n_total, Hq] or NULL.
  * Errors: TG_ERR_INVALID_ARG (null pointer, bad sizes, misaligned q/k/v),
  *   TG_ERR_UNSUPPORTED (D or G outside the list), TG_ERR_CUDA.  A malformed
- *   tree sets TG_ERR_DEVICE_TREE; its rows of `out` are then left unwritten.
+ *   tree sets TG_ERR_DEVICE_TREE; its rows of `out` and `lse_out` are then
+ *   undefined (computed with every tree slot masked).
  */
 int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
                         const int32_t* prefix_len, const int32_t* parent,

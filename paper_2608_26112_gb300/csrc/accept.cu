@@ -24,17 +24,18 @@ namespace tg {
 namespace {
 
 struct AcceptSmem {
-  uint64_t red[8];
-  uint64_t peer_key;
-  int tree, off, n, last;
+  float red_v[8];
+  uint64_t recv_key[16];  // leader only: per-CTA (max, first position) keys of the row
+  int minpos;
+  int tree, off, n, last, bad;
   int par[256];
   int am[256];
+  int tok[256];
   uint32_t key[8];
-  int bad;
 };
 
 template <typename T, bool kAligned>
-__global__ void __launch_bounds__(kScanThreads) accept_kernel(AcceptArgs a, int row_base) {
+__global__ void __launch_bounds__(kScanThreads, 4) accept_kernel(AcceptArgs a, int row_base) {
   __shared__ AcceptSmem sm;
   cg::cluster_group cluster = cg::this_cluster();
   const int C = (int)cluster.num_blocks();
@@ -43,6 +44,7 @@ __global__ void __launch_bounds__(kScanThreads) accept_kernel(AcceptArgs a, int 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int VW = ScanTraits<T>::kVW;
   const int V = a.V;
+  cluster_arrive_relaxed();
   const int per = ((V + C - 1) / C + VW - 1) / VW * VW;
   const int c0 = min(V, crank * per);
   const int c1 = min(V, c0 + per);
@@ -50,32 +52,33 @@ __global__ void __launch_bounds__(kScanThreads) accept_kernel(AcceptArgs a, int 
 
   uint4 buf[kScanVecs];
   scan_load<T, kAligned>(rowp, c0, c1, buf);
-  float tmax;
-  int tpos;
-  scan_thread_max<T>(buf, c0, c1, tmax, tpos);
-  uint64_t key = (tpos < 0) ? 0ull : make_key(tmax, (uint32_t)tpos);
-  key = warp_max_u64(key);
-  if (lane == 0) sm.red[warp] = key;
+  if (tid == 0) sm.minpos = 0x7FFFFFFF;
+  // chunk max, then the lowest position holding it (only threads that hold it search)
+  const float tmax = scan_thread_max<T>(buf);
+  const float wm = warp_max_f32(tmax);
+  if (lane == 0) sm.red_v[warp] = wm;
   __syncthreads();
-  if (tid == 0) {
-    uint64_t m = sm.red[0];
+  float cmax = sm.red_v[0];
 #pragma unroll
-    for (int w = 1; w < 8; ++w) m = sm.red[w] > m ? sm.red[w] : m;
-    sm.peer_key = m;
+  for (int w = 1; w < 8; ++w) cmax = fmaxf(cmax, sm.red_v[w]);
+  if (tmax == cmax && c0 + (int)tid * VW < c1) {
+    const int fp = scan_first_pos<T>(buf, c0, c1, cmax);
+    if (fp != 0x7FFFFFFF) atomicMin(&sm.minpos, fp);
   }
-  cluster.sync();
-  uint64_t best = 0;
-  if (crank == 0 && tid == 0) {
-    for (int c = 0; c < C; ++c) {
-      const uint64_t kc = cluster.map_shared_rank(&sm, c)->peer_key;
-      best = kc > best ? kc : best;
-    }
+  __syncthreads();
+  cluster_wait();
+  if (tid == 0) {
+    const int mp = sm.minpos;
+    cluster.map_shared_rank(&sm, 0)->recv_key[crank] =
+        (mp == 0x7FFFFFFF) ? 0ull : make_key(cmax, (uint32_t)mp);
   }
   cluster.sync();
   if (crank != 0) return;
 
   // leader: publish the argmax, take a ticket for the row's tree
   if (tid == 0) {
+    uint64_t best = 0;
+    for (int c = 0; c < C; ++c) best = sm.recv_key[c] > best ? sm.recv_key[c] : best;
     a.am[row] = (int32_t)key_index(best);
     // tree of this row: last b with node_off[b] <= row
     int lo = 0, hi = a.B - 1;
@@ -100,15 +103,15 @@ __global__ void __launch_bounds__(kScanThreads) accept_kernel(AcceptArgs a, int 
     if (sm.bad) raise_status(a.status, kStTree);
   }
   __syncthreads();
-  if (!sm.last) return;
+  if (!sm.last || sm.bad) return;
 
   // ---- walk of tree b (this CTA saw every row of the tree finish)
   const int b = sm.tree, off = sm.off, n = sm.n;
-  if (sm.bad) return;
   int v_par = -1;
   if (tid < n) {
     v_par = a.parent[off + tid];
     sm.par[tid] = v_par;
+    sm.tok[tid] = a.token[off + tid];
     sm.am[tid] = __ldcg(&a.am[off + tid]);
   }
   const bool bad = (tid < n) && (tid == 0 ? (v_par != -1) : (v_par < 0 || v_par >= tid));
@@ -117,13 +120,13 @@ __global__ void __launch_bounds__(kScanThreads) accept_kernel(AcceptArgs a, int 
     return;
   }
   uint32_t wkey = 0;
-  int depth = 0;
   if (tid < n) {
     bool full = true;
+    int depth = 0;
     int v = tid;
     while (v != 0) {  // parent[v] < v: at most v steps
       const int p = sm.par[v];
-      full = full && (a.token[off + v] == sm.am[p]);
+      full = full && (sm.tok[v] == sm.am[p]);
       v = p;
       ++depth;
     }

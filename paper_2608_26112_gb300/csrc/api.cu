@@ -110,7 +110,7 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
   const int G = Hq / Hkv;
   if (D != 64 && D != 128) return TG_ERR_UNSUPPORTED;
   if (G != 1 && G != 2 && G != 4 && G != 8) return TG_ERR_UNSUPPORTED;
-  if ((long long)B * Hkv > 65535 || (long long)B * Hkv * S_max + 128 >= (1ll << 31))
+  if ((long long)B * Hkv > 65535 || (long long)B * Hkv * S_max + 128 * 32 >= (1ll << 31))
     return TG_ERR_UNSUPPORTED;
   if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out))
     return TG_ERR_INVALID_ARG;
@@ -148,7 +148,7 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
   a.lse_out = lse_out;
   a.status = st;
   const int mtiles = (G * max_nodes + 127) / 128;
-  const int splits = tree_attn_pick_splits(B, Hkv, mtiles, S_max, device_sm_count());
+  const int splits = tree_attn_pick_splits(D, B, Hkv, mtiles, S_max, device_sm_count());
   return launch_tree_attn(tq, tk, tv, a, splits, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? TG_OK
              : TG_ERR_CUDA;

@@ -22,7 +22,7 @@ struct AttnArgs {
 cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                              const CUtensorMap& tm_v, const AttnArgs& a, int kv_splits,
                              cudaStream_t s);
-int tree_attn_pick_splits(int B, int Hkv, int mtiles, int S_max, int num_sms);
+int tree_attn_pick_splits(int D, int B, int Hkv, int mtiles, int S_max, int num_sms);
 
 struct TopkArgs {
   const void* logits;

@@ -6,7 +6,13 @@
 // CTA keeps 32 KB of reads in flight and the whole grid saturates HBM with a
 // single pass.  Element (i, j) of a thread is vector i, lane j, at row
 // position c0 + (i * 256 + threadIdx.x) * VW + j: positions increase with
-// (i, j), so "first in scan order" is "lowest token id".
+// (i, j), so "first in scan order" is "lowest token id".  Positions past c1
+// are loaded as -inf, which no max, exp or threshold test can pick.
+//
+// The per-element work is kept to what the math needs: the thread max uses
+// packed bf16x2 max (half an instruction per element), the exp-sum is taken
+// relative to the thread's own max (no block barrier in between), and
+// positions are only materialised for the few elements that can win.
 #pragma once
 
 #include "common.cuh"
@@ -15,6 +21,8 @@ namespace tg {
 
 constexpr int kScanThreads = 256;
 constexpr int kScanVecs = 8;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
 
 template <typename T>
 struct ScanTraits;
@@ -51,6 +59,10 @@ __device__ __forceinline__ float vec_elem<float>(const uint4& v, int j) {
   return __uint_as_float(vec_word(v, j));
 }
 
+__device__ __forceinline__ int scan_pos(int c0, int i, int j, int vw) {
+  return c0 + (i * kScanThreads + (int)threadIdx.x) * vw + j;
+}
+
 // Load this thread's elements of [c0, c1); positions past c1 read as -inf.
 // kAligned: the row start is 16-byte aligned (c0 is a multiple of VW).
 template <typename T, bool kAligned>
@@ -59,7 +71,7 @@ __device__ __forceinline__ void scan_load(const T* __restrict__ row, int c0, int
   constexpr int VW = ScanTraits<T>::kVW;
 #pragma unroll
   for (int i = 0; i < kScanVecs; ++i) {
-    const int pos = c0 + (i * kScanThreads + (int)threadIdx.x) * VW;
+    const int pos = scan_pos(c0, i, 0, VW);
     if (kAligned && pos + VW <= c1) {
       buf[i] = ld_stream_v4(row + pos);
     } else {
@@ -89,27 +101,82 @@ __device__ __forceinline__ void scan_load(const T* __restrict__ row, int c0, int
   }
 }
 
-// Largest element of this thread and its lowest position (-inf elements
-// count; a thread without elements returns pos = -1).
+// Largest element of this thread (-inf if it has none).
 template <typename T>
-__device__ __forceinline__ void scan_thread_max(const uint4 (&buf)[kScanVecs], int c0, int c1,
-                                                float& vmax, int& pmax) {
-  constexpr int VW = ScanTraits<T>::kVW;
-  vmax = __int_as_float(0xff800000);
-  pmax = -1;
+__device__ __forceinline__ float scan_thread_max(const uint4 (&buf)[kScanVecs]);
+template <>
+__device__ __forceinline__ float scan_thread_max<__nv_bfloat16>(const uint4 (&buf)[kScanVecs]) {
+  __nv_bfloat162 m[4];
 #pragma unroll
-  for (int i = 0; i < kScanVecs; ++i) {
-    const int base = c0 + (i * kScanThreads + (int)threadIdx.x) * VW;
-#pragma unroll
-    for (int j = 0; j < VW; ++j) {
-      const float v = vec_elem<T>(buf[i], j);
-      const int pos = base + j;
-      if (pos < c1 && (pmax < 0 || v > vmax)) {
-        vmax = v;
-        pmax = pos;
-      }
-    }
+  for (int w = 0; w < 4; ++w) {
+    uint32_t x = vec_word(buf[0], w);
+    m[w] = *reinterpret_cast<__nv_bfloat162*>(&x);
   }
+#pragma unroll
+  for (int i = 1; i < kScanVecs; ++i)
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      uint32_t x = vec_word(buf[i], w);
+      m[w] = __hmax2(m[w], *reinterpret_cast<__nv_bfloat162*>(&x));
+    }
+  const __nv_bfloat162 a = __hmax2(__hmax2(m[0], m[1]), __hmax2(m[2], m[3]));
+  return fmaxf(__low2float(a), __high2float(a));
+}
+template <>
+__device__ __forceinline__ float scan_thread_max<float>(const uint4 (&buf)[kScanVecs]) {
+  float m = __uint_as_float(buf[0].x);
+#pragma unroll
+  for (int i = 0; i < kScanVecs; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) m = fmaxf(m, __uint_as_float(vec_word(buf[i], j)));
+  return m;
+}
+
+// sum_t 2^((x_t - m) * log2 e) over this thread's elements, m = its max
+template <typename T>
+__device__ __forceinline__ float scan_thread_sumexp(const uint4 (&buf)[kScanVecs], float m) {
+  if (m == __int_as_float(0xff800000)) return 0.f;
+  constexpr int VW = ScanTraits<T>::kVW;
+  const float mb = -m * kLog2e;
+  float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+  for (int i = 0; i < kScanVecs; ++i)
+#pragma unroll
+    for (int j = 0; j < VW; j += 2) {
+      s0 += ex2(fmaf(vec_elem<T>(buf[i], j), kLog2e, mb));
+      s1 += ex2(fmaf(vec_elem<T>(buf[i], j + 1), kLog2e, mb));
+    }
+  return s0 + s1;
+}
+
+// Lowest position in [c0, c1) whose value equals v (INT_MAX if none).
+template <typename T>
+__device__ __forceinline__ int scan_first_pos(const uint4 (&buf)[kScanVecs], int c0, int c1,
+                                              float v) {
+  constexpr int VW = ScanTraits<T>::kVW;
+  int best = 0x7FFFFFFF;
+#pragma unroll
+  for (int i = kScanVecs - 1; i >= 0; --i)
+#pragma unroll
+    for (int j = VW - 1; j >= 0; --j) {
+      const int pos = scan_pos(c0, i, j, VW);
+      if (pos < c1 && vec_elem<T>(buf[i], j) == v) best = pos;
+    }
+  return best;
+}
+
+// Combine two (max, sum of 2^(x - max)) pairs.
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
+  const float NEG_INF = __int_as_float(0xff800000);
+  const float M = fmaxf(m, m2);
+  if (M == NEG_INF) {
+    m = M;
+    s = 0.f;
+    return;
+  }
+  s = (m == NEG_INF ? 0.f : s * ex2((m - M) * kLog2e)) +
+      (m2 == NEG_INF ? 0.f : s2 * ex2((m2 - M) * kLog2e));
+  m = M;
 }
 
 }  // namespace tg

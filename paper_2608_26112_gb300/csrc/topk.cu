@@ -4,17 +4,22 @@
 //
 // Grid (C, rows) with clusters of C CTAs along x: the C CTAs of a cluster
 // split one row.  Each CTA
-//   1. stages its chunk in registers (rowscan.cuh),
-//   2. reduces the chunk max m_c and sum_t exp(l_t - m_c),
-//   3. finds an exact threshold key: the k-th largest of the 256 per-thread
-//      maxima (a warp bitonic sort, then a rank count over 8 * k keys).  At
-//      least k elements reach it and only the k threads owning the top-k
-//      maxima can hold elements above it, so at most 64 * k candidates pass,
-//   4. collects the candidates in shared memory and ranks them to its local
-//      top-k (64-bit keys: value desc, token asc - exact on ties).
-// The cluster leader then pulls every CTA's (m_c, s_c, top-k) over DSMEM,
-// merges them into lse and the row's top-k, and writes the outputs.  No
-// global scratch and no second launch.
+//   1. stages its chunk in registers and takes per-thread (max, sum of
+//      exp(x - max)) - packed bf16x2 max, one exp per element;
+//   2. sorts the 256 thread maxima per warp and picks the value threshold
+//      t = the largest value v with at least k thread maxima >= v.  At
+//      least k elements reach t, and only threads whose max reaches t can
+//      hold elements that do, so candidates are collected by a handful of
+//      threads only;
+//   3. ranks the candidates by 64-bit keys (value desc, token asc - exact
+//      on ties) into its local top-k.  Heavily tied chunks can overflow the
+//      candidate buffer; they fall back to an exact key threshold (the k-th
+//      largest per-thread (max, first position) key), which bounds the
+//      candidates by 64 * k;
+//   4. pushes (max, sum, top-k) into the cluster leader's shared memory
+//      (DSMEM stores) and meets the cluster barrier once.
+// The leader merges the C partials into lse and the row's top-k and writes
+// the outputs.  No global scratch and no second launch.
 #include <cooperative_groups.h>
 
 #include "launch.h"
@@ -26,37 +31,35 @@ namespace tg {
 namespace {
 
 constexpr int kMaxK = 32;
-constexpr int kCandMax = kMaxK * kScanVecs * 8;  // 64 elements/thread * k
+constexpr int kCandMax = 2048;  // >= 64 elements/thread * kMaxK
 constexpr int kMaxCluster = 16;
-constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kLn2 = 0.6931471805599453f;
+static_assert(kCandMax >= kScanVecs * 8 * kMaxK, "exact fallback must fit the buffer");
 
 struct TopkSmem {
   uint64_t cand[kCandMax];
-  uint64_t warp_top[8 * kMaxK];
   uint64_t top[kMaxK];
-  uint64_t merged[kMaxCluster * kMaxK];
-  float merged_m[kMaxCluster];
-  float merged_s[kMaxCluster];
-  float red_f[8];
-  float part_m, part_s;
-  uint64_t thr;
+  uint64_t recv_top[kMaxCluster * kMaxK];  // leader only: partials pushed by the cluster
+  float recv_m[kMaxCluster];
+  float recv_s[kMaxCluster];
+  float warp_v[8 * kMaxK];
+  uint64_t warp_k[8 * kMaxK];
+  float red_m[8], red_s[8];
+  uint32_t thr_ord;
+  uint64_t thr_key;
   int ncand;
-  int bad_row;
+  float lse;
 };
 
-// descending bitonic sort of one 64-bit key per lane; lane j ends with the
-// j-th largest
-__device__ __forceinline__ uint64_t warp_sort_desc(uint64_t x) {
+// descending bitonic sort of one value per lane; lane j ends with the j-th largest
+template <typename K>
+__device__ __forceinline__ K warp_sort_desc(K x) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
   for (int size = 2; size <= 32; size <<= 1) {
 #pragma unroll
     for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      const uint64_t y = __shfl_xor_sync(0xffffffffu, x, stride);
-      const bool asc_block = (lane & size) == 0;
-      const bool lower = (lane & stride) == 0;
-      const bool take_max = (lower == asc_block);
+      const K y = __shfl_xor_sync(0xffffffffu, x, stride);
+      const bool take_max = (((lane & stride) == 0) == ((lane & size) == 0));
       x = take_max ? (x > y ? x : y) : (x < y ? x : y);
     }
   }
@@ -64,7 +67,7 @@ __device__ __forceinline__ uint64_t warp_sort_desc(uint64_t x) {
 }
 
 template <typename T, bool kAligned>
-__global__ void __launch_bounds__(kScanThreads) expand_topk_kernel(TopkArgs a) {
+__global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a) {
   __shared__ TopkSmem sm;
   cg::cluster_group cluster = cg::this_cluster();
   const int C = (int)cluster.num_blocks();
@@ -73,6 +76,7 @@ __global__ void __launch_bounds__(kScanThreads) expand_topk_kernel(TopkArgs a) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int k = a.k;
   const int V = a.V;
+  constexpr int VW = ScanTraits<T>::kVW;
 
   // physical row (uniform over the cluster: every CTA reads the same index)
   int r = row;
@@ -81,7 +85,7 @@ __global__ void __launch_bounds__(kScanThreads) expand_topk_kernel(TopkArgs a) {
     if (crank == 0 && tid == 0) raise_status(a.status, kStIndex);
     return;
   }
-  constexpr int VW = ScanTraits<T>::kVW;
+  cluster_arrive_relaxed();
   const int per = ((V + C - 1) / C + VW - 1) / VW * VW;
   const int c0 = min(V, crank * per);
   const int c1 = min(V, c0 + per);
@@ -89,135 +93,130 @@ __global__ void __launch_bounds__(kScanThreads) expand_topk_kernel(TopkArgs a) {
 
   uint4 buf[kScanVecs];
   scan_load<T, kAligned>(rowp, c0, c1, buf);
-
   if (tid == 0) {
-    sm.thr = 0;
+    sm.thr_ord = 0u;
     sm.ncand = 0;
   }
-  if (tid < kMaxK) sm.top[tid] = 0;
+  if (tid < kMaxK) sm.top[tid] = 0ull;
 
-  // 1. thread max (first position on ties) and chunk max
-  float tmax;
-  int tpos;
-  scan_thread_max<T>(buf, c0, c1, tmax, tpos);
-  float wm = warp_max_f32(tmax);
-  if (lane == 0) sm.red_f[warp] = wm;
-  __syncthreads();
-  float m_c = sm.red_f[0];
+  // 1. per-thread max and exp-sum, warp-combined
+  const float tmax = scan_thread_max<T>(buf);
+  float m = tmax, s = scan_thread_sumexp<T>(buf, tmax);
 #pragma unroll
-  for (int w = 1; w < 8; ++w) m_c = fmaxf(m_c, sm.red_f[w]);
-
-  // 2. sum of exp(l - m_c)
-  float ssum = 0.f;
-  if (m_c != __int_as_float(0xff800000)) {
-    const float mb = -m_c * kLog2e;
-#pragma unroll
-    for (int i = 0; i < kScanVecs; ++i) {
-#pragma unroll
-      for (int j = 0; j < VW; ++j) ssum += ex2(fmaf(vec_elem<T>(buf[i], j), kLog2e, mb));
-    }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    lse_merge(m, s, m2, s2);
   }
-  ssum = warp_sum_f32(ssum);
-  __syncthreads();  // red_f reuse
-  if (lane == 0) sm.red_f[warp] = ssum;
-
-  // 3. threshold = k-th largest per-thread max key
-  const uint64_t tkey = (tpos < 0) ? 0ull : make_key(tmax, (uint32_t)tpos);
-  const uint64_t sorted = warp_sort_desc(tkey);
-  if (lane < k) sm.warp_top[warp * k + lane] = sorted;
-  __syncthreads();
-  if (tid == 0) {
-    float s = 0.f;
-#pragma unroll
-    for (int w = 0; w < 8; ++w) s += sm.red_f[w];
-    sm.part_m = m_c;
-    sm.part_s = s;
+  // 2. value threshold from the sorted thread maxima
+  const float sv = warp_sort_desc<float>(tmax);
+  if (lane < k) sm.warp_v[warp * k + lane] = sv;
+  if (lane == 0) {
+    sm.red_m[warp] = m;
+    sm.red_s[warp] = s;
   }
+  __syncthreads();
   if (tid < 8 * k) {
-    const uint64_t mine = sm.warp_top[tid];
-    int rank = 0;
-    for (int i = 0; i < 8 * k; ++i) rank += (sm.warp_top[i] > mine) ? 1 : 0;
-    if (mine != 0ull && rank == k - 1) sm.thr = mine;
+    const float v = sm.warp_v[tid];
+    int ge = 0;
+    for (int i = 0; i < 8 * k; ++i) ge += (sm.warp_v[i] >= v) ? 1 : 0;
+    if (ge >= k && v == v) atomicMax(&sm.thr_ord, ord_f32(v));
   }
   __syncthreads();
-
-  // 4. candidates: elements whose key reaches the threshold
-  {
-    const uint64_t thr = sm.thr;
-    const bool take_all = (thr == 0ull);
-    const float tv = key_value(thr);
-    const int tp = (int)key_index(thr);
+  const float tv = unord_f32(sm.thr_ord);
+  // 3. candidates (only threads whose max reaches the threshold have any)
+  if (tmax >= tv) {
 #pragma unroll
-    for (int i = 0; i < kScanVecs; ++i) {
-      const int base = c0 + (i * kScanThreads + tid) * VW;
+    for (int i = 0; i < kScanVecs; ++i)
 #pragma unroll
       for (int j = 0; j < VW; ++j) {
         const float v = vec_elem<T>(buf[i], j);
-        const int pos = base + j;
-        if (pos < c1 && (take_all || v > tv || (v == tv && pos <= tp))) {
+        const int pos = scan_pos(c0, i, j, VW);
+        if (pos < c1 && v >= tv) {
           const int slot = atomicAdd(&sm.ncand, 1);
           if (slot < kCandMax) sm.cand[slot] = make_key(v, (uint32_t)pos);
         }
       }
-    }
   }
   __syncthreads();
-  {
-    const int nc = min(sm.ncand, kCandMax);
-    for (int i = tid; i < nc; i += kScanThreads) {
-      const uint64_t mine = sm.cand[i];
+  int nc = sm.ncand;
+  if (nc > kCandMax) {
+    // heavy ties: exact key threshold = k-th largest (thread max, first position)
+    __syncthreads();  // every thread has read ncand before it is reset below
+    const int fp = (c0 + (int)tid * VW >= c1) ? 0x7FFFFFFF : scan_first_pos<T>(buf, c0, c1, tmax);
+    const uint64_t tk = (fp == 0x7FFFFFFF) ? 0ull : make_key(tmax, (uint32_t)fp);
+    const uint64_t sk = warp_sort_desc<uint64_t>(tk);
+    if (lane < k) sm.warp_k[warp * k + lane] = sk;
+    if (tid == 0) {
+      sm.thr_key = 0ull;
+      sm.ncand = 0;
+    }
+    __syncthreads();
+    if (tid < 8 * k) {
+      const uint64_t mine = sm.warp_k[tid];
       int rank = 0;
-      for (int j = 0; j < nc; ++j) rank += (sm.cand[j] > mine) ? 1 : 0;
-      if (rank < k) sm.top[rank] = mine;
+      for (int i = 0; i < 8 * k; ++i) rank += (sm.warp_k[i] > mine) ? 1 : 0;
+      if (mine != 0ull && rank == k - 1) sm.thr_key = mine;
     }
+    __syncthreads();
+    const uint64_t thr = sm.thr_key;
+    if (tk >= thr && tk != 0ull) {
+#pragma unroll
+      for (int i = 0; i < kScanVecs; ++i)
+#pragma unroll
+        for (int j = 0; j < VW; ++j) {
+          const int pos = scan_pos(c0, i, j, VW);
+          const uint64_t key = make_key(vec_elem<T>(buf[i], j), (uint32_t)pos);
+          if (pos < c1 && key >= thr) {
+            const int slot = atomicAdd(&sm.ncand, 1);
+            if (slot < kCandMax) sm.cand[slot] = key;
+          }
+        }
+    }
+    __syncthreads();
+    nc = min(sm.ncand, kCandMax);
   }
+  for (int i = tid; i < nc; i += kScanThreads) {
+    const uint64_t mine = sm.cand[i];
+    int rank = 0;
+    for (int j = 0; j < nc; ++j) rank += (sm.cand[j] > mine) ? 1 : 0;
+    if (rank < k) sm.top[rank] = mine;
+  }
+  __syncthreads();
 
-  // 5. cluster merge at rank 0
-  cluster.sync();
-  if (crank == 0) {
-    for (int t = tid; t < C * k; t += kScanThreads) {
-      const TopkSmem* peer = cluster.map_shared_rank(&sm, t / k);
-      sm.merged[t] = peer->top[t % k];
-    }
-    if (tid < C) {
-      const TopkSmem* peer = cluster.map_shared_rank(&sm, tid);
-      sm.merged_m[tid] = peer->part_m;
-      sm.merged_s[tid] = peer->part_s;
-    }
+  // 4. push the partial into the leader's shared memory
+  cluster_wait();
+  TopkSmem* lead = cluster.map_shared_rank(&sm, 0);
+  if (tid < k) lead->recv_top[crank * k + tid] = sm.top[tid];
+  if (tid == 0) {
+    float M = sm.red_m[0], S = sm.red_s[0];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) lse_merge(M, S, sm.red_m[w], sm.red_s[w]);
+    lead->recv_m[crank] = M;
+    lead->recv_s[crank] = S;
   }
   cluster.sync();
   if (crank != 0) return;
 
-  __shared__ float lse_s;
+  // ---- leader: merge the C partials
   if (tid == 0) {
-    float M = sm.merged_m[0];
-    for (int c = 1; c < C; ++c) M = fmaxf(M, sm.merged_m[c]);
-    float lse;
-    if (M == __int_as_float(0xff800000)) {
-      lse = M;
-    } else {
-      float S = 0.f;
-      for (int c = 0; c < C; ++c) {
-        const float mc = sm.merged_m[c];
-        if (mc != __int_as_float(0xff800000)) S += sm.merged_s[c] * ex2((mc - M) * kLog2e);
-      }
-      lse = M + log2f(S) * kLn2;
-    }
-    lse_s = lse;
+    float M = sm.recv_m[0], S = sm.recv_s[0];
+    for (int c = 1; c < C; ++c) lse_merge(M, S, sm.recv_m[c], sm.recv_s[c]);
+    const float lse = (M == __int_as_float(0xff800000)) ? M : M + log2f(S) * kLn2;
+    sm.lse = lse;
     if (a.lse_out) a.lse_out[row] = lse;
   }
-  __syncthreads();
   for (int t = tid; t < C * k; t += kScanThreads) {
-    const uint64_t mine = sm.merged[t];
+    const uint64_t mine = sm.recv_top[t];
     int rank = 0;
-    for (int j = 0; j < C * k; ++j) rank += (sm.merged[j] > mine) ? 1 : 0;
-    if (rank < k) sm.top[rank] = mine;  // own top[] is no longer read by peers
+    for (int j = 0; j < C * k; ++j) rank += (sm.recv_top[j] > mine) ? 1 : 0;
+    if (rank < k) sm.top[rank] = mine;
   }
   __syncthreads();
   if (tid < k) {
     const uint64_t key = sm.top[tid];
     const float v = key_value(key);
-    const float lse = lse_s;
+    const float lse = sm.lse;
     const float lp = (lse == __int_as_float(0xff800000)) ? lse : (v - lse);
     const size_t o = (size_t)row * k + tid;
     a.tok[o] = (int32_t)key_index(key);
@@ -237,10 +236,12 @@ cudaError_t launch_topk_t(const TopkArgs& a, int C, cudaStream_t s) {
     TopkArgs b = a;
     const int nr = min(65535, a.rows - r0);
     b.rows = nr;
-    if (b.row_idx) b.row_idx += r0;
-    else b.logits = static_cast<const char*>(a.logits) +
-                    (size_t)r0 * (size_t)a.ld * (a.is_bf16 ? 2 : 4);
-    if (!b.row_idx) b.logit_rows = a.logit_rows - r0;
+    if (b.row_idx) {
+      b.row_idx += r0;
+    } else {
+      b.logits = static_cast<const char*>(a.logits) + (size_t)r0 * (size_t)a.ld * (a.is_bf16 ? 2 : 4);
+      b.logit_rows = a.logit_rows - r0;
+    }
     b.parent_score += r0;
     b.tok += (size_t)r0 * a.k;
     b.logprob += (size_t)r0 * a.k;
@@ -272,11 +273,10 @@ int scan_cluster_size(int V, int is_bf16, int rows, int num_sms) {
   const int epc = is_bf16 ? scan_elems_per_cta<__nv_bfloat16>() : scan_elems_per_cta<float>();
   int C = (V + epc - 1) / epc;
   if (C < 1) C = 1;
-  // with few rows, spread each row over more CTAs (at least ~1 CTA per SM)
   const int vw = is_bf16 ? 8 : 4;
   while (C < kMaxCluster && (long long)rows * C < num_sms && (V + 2 * C - 1) / (2 * C) >= 256 * vw)
     C *= 2;
-  return C > kMaxCluster ? -1 : C;
+  return C > kMaxCluster ? kMaxCluster : C;
 }
 
 cudaError_t launch_expand_topk(const TopkArgs& a, cudaStream_t s) {

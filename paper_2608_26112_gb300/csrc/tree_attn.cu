@@ -6,22 +6,29 @@
 // row index u*G + g, so the tile is a dense 128 x D bf16 operand: a single
 // 3-D TMA box {64, G, 128/G} of q gathers it.  The key axis (prefix
 // [0, P) followed by the tree slots [P, P+n)) is cut into 128-key tiles;
-// the S_kv CTAs of a thread-block cluster split those tiles and combine
-// their partial (max, sum, O) rows over DSMEM at the end, so nothing but
-// the final bf16 output and the lse touch global memory.
+// the S_kv CTAs of a thread-block cluster take the tiles round-robin (split
+// s: tiles s, s + S_kv, ...), so each CTA can start its first K/V copies
+// before it has read anything from global memory.
 //
-// Warp roles (192 threads, one CTA per SM):
-//   warp 0      TMA producer: Q once, then K and V tiles into a 2-stage ring;
-//   warp 1      TMEM owner and MMA issuer: S = Q K^T (M=128, N=128, K=D) and
-//               O += P V (M=128, N=D, K=128), bf16 in, fp32 accumulate in
-//               TMEM, completion signalled by tcgen05.commit on mbarriers;
-//   warps 2..5  softmax: one query row per thread (TMEM lane = row), read
-//               S with tcgen05.ld, apply the ancestor mask from a per-node
-//               bitmask in shared memory, online max / sum in base 2, write
-//               P as bf16 into the swizzled operand layout, rescale O in
-//               TMEM when the running max grows; finally the combine.
-// The MMA thread issues S(i+1) before PV(i), so the softmax of tile i+1
-// overlaps the PV product of tile i.  Every mbarrier wait is bounded.
+// Warp roles (320 threads, one CTA per SM):
+//   warp 0      TMA producer: K and V tiles into a 2-stage ring, Q once;
+//   warp 1      TMEM owner and MMA issuer: S = Q K^T (M=128, N=128, K=D) into
+//               one of two TMEM buffers and O += P V (M=128, N=D, K=128),
+//               bf16 in, fp32 accumulate, completion signalled by
+//               tcgen05.commit on mbarriers.  Pipe order S(0) S(1) PV(0)
+//               S(2) PV(1) ...: S(i+1) runs while the softmax of tile i runs;
+//   warps 2..9  softmax: two threads per query row (TMEM lane = row), each
+//               owning half of the 128 key columns and half of O's columns.
+//               They read S with tcgen05.ld, apply the ancestor mask from a
+//               per-node bitmask in shared memory, exchange the row max
+//               through shared memory, keep a base-2 online max / sum, write
+//               P as bf16 into the swizzled operand layout, and rescale O in
+//               TMEM when the running max grows.
+// Split combine: each CTA stages its partial rows (O, max, sum) in shared
+// memory; between two cluster barriers every CTA reads the S_kv partials of
+// the rows it owns from its peers' shared memory (DSMEM) and writes the
+// normalised rows.  With a single split the rows are normalised and written
+// straight from TMEM.  Every mbarrier wait is bounded.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -32,16 +39,18 @@ namespace cg = cooperative_groups;
 namespace tg {
 namespace {
 
-constexpr int kBM = 128;     // query rows per tile (TMEM lanes)
-constexpr int kBN = 128;     // keys per KV tile
-constexpr int kStages = 2;   // K/V ring depth
-constexpr int kThreads = 192;
-constexpr int kAncWords = 9; // 256 tree slots + one zero word
+constexpr int kBM = 128;      // query rows per tile (TMEM lanes)
+constexpr int kBN = 128;      // keys per KV tile
+constexpr int kStages = 2;    // K and V ring depth
+constexpr int kSoftmaxThreads = 256;
+constexpr int kThreads = 64 + kSoftmaxThreads;
+constexpr int kAncWords = 9;  // 256 tree slots + one zero word
 constexpr int kRegion = 128 * 128;  // 128 rows x 128 bytes: one swizzled operand region
+constexpr int kMaxSplits = 8;
 constexpr float kLn2 = 0.6931471805599453f;
 
-enum { BAR_KV_FULL = 0, BAR_KV_EMPTY = 2, BAR_Q_FULL = 4, BAR_S_FULL = 5, BAR_P_FULL = 6,
-       BAR_O_DONE = 7, kNumBars = 8 };
+enum { BAR_KV_FULL = 0, BAR_KV_EMPTY = 2, BAR_Q_FULL = 4, BAR_S_FULL = 5 /* 2 buffers */,
+       BAR_P_FULL = 7, BAR_O_DONE = 8, kNumBars = 9 };
 
 constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
@@ -54,24 +63,25 @@ struct Layout {
   static constexpr int kOffK = kOffQ + kQBytes;
   static constexpr int kOffV = kOffK + kStages * kKVBytes;
   static constexpr int kOffP = kOffV + kStages * kKVBytes;
-  static constexpr int kOffAnc = kOffP + kPBytes;                  // (kBM + 1) rows
+  static constexpr int kTileEnd = kOffP + kPBytes;
+  static constexpr int kOffAnc = kTileEnd;                            // (kBM + 1) rows
   static constexpr int kOffPar = align_up(kOffAnc + (kBM + 1) * kAncWords * 4, 16);
-  static constexpr int kOffM = align_up(kOffPar + 256 * 4, 16);
-  static constexpr int kOffL = align_up(kOffM + kBM * 4, 16);
-  static constexpr int kOffBar = align_up(kOffL + kBM * 4, 16);    // mbarriers: 8-byte aligned
-  static constexpr int kOffTmem = align_up(kOffBar + kNumBars * 8, 16);
-  static constexpr int kBytes = kOffTmem + 16;
-  static constexpr int kAlloc = kBytes + 1024;                     // 1024-byte alignment slack
-  // fp32 O staging for the combine, padded rows, reusing the K/V ring
-  static constexpr int kOStride = D + 4;
-  static constexpr int kOffO = kOffK;
-  static_assert(kBM * kOStride * 4 <= 2 * kStages * kKVBytes, "O staging must fit in K/V ring");
+  static constexpr int kOffRedMax = align_up(kOffPar + 256 * 4, 16); // [2 parity][2 half][kBM]
+  static constexpr int kOffRedL = align_up(kOffRedMax + 4 * kBM * 4, 16);  // [2 half][kBM]
+  static constexpr int kOffBar = align_up(kOffRedL + 2 * kBM * 4, 16);     // mbarriers
+  static constexpr int kOffMisc = align_up(kOffBar + kNumBars * 8, 16);    // tmem addr, flag
+  static constexpr int kBytes = kOffMisc + 16;
+  static constexpr int kAlloc = kBytes + 1024;                       // 1024-byte alignment slack
+  // Partial rows of the combine, written once every MMA of the CTA is done,
+  // over the Q / K tiles: a row is [O (D fp32) | m (base 2) | l | 2 pad].
+  static constexpr int kRowFloats = D + 4;
+  static constexpr int kOffStage = 0;
+  static_assert(kOffStage + kBM * kRowFloats * 4 <= kTileEnd, "staging fits the tiles");
   static_assert(kAlloc <= 227 * 1024, "shared memory budget");
   static_assert(kOffQ % 1024 == 0 && kOffK % 1024 == 0 && kOffV % 1024 == 0 && kOffP % 1024 == 0,
                 "128-byte-swizzled operand tiles need 1024-byte alignment");
-  static_assert(kOffBar % 8 == 0 && kOffTmem % 4 == 0 && kOffM % 16 == 0 && kOffL % 16 == 0,
-                "mbarrier / scalar alignment");
-  static_assert((kOStride * 4) % 16 == 0, "float4 rows of the O staging");
+  static_assert(kOffBar % 8 == 0 && kOffMisc % 16 == 0, "mbarrier / scalar alignment");
+  static_assert((kRowFloats * 4) % 16 == 0, "float4 staging rows");
 };
 
 // 32 mask bits of one node for tree slots [b0, b0 + 32): slot < 0 is the
@@ -100,12 +110,18 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
+// barrier among the 256 softmax threads only (id 1; id 0 is __syncthreads)
+__device__ __forceinline__ void softmax_bar() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                      const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const AttnArgs a) {
   using L = Layout<D>;
+  constexpr int DH = D / 2;  // O columns per softmax thread
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -119,102 +135,110 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   int* par_s = reinterpret_cast<int*>(smem + L::kOffPar);
   uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + L::kOffAnc);
-  float* m_s = reinterpret_cast<float*>(smem + L::kOffM);
-  float* l_s = reinterpret_cast<float*>(smem + L::kOffL);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kOffTmem);
+  float* red_max = reinterpret_cast<float*>(smem + L::kOffRedMax);
+  float* red_l = reinterpret_cast<float*>(smem + L::kOffRedL);
+  float* stage_rows = reinterpret_cast<float*>(smem + L::kOffStage);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kOffMisc);
+  int* bad_flag = reinterpret_cast<int*>(smem + L::kOffMisc + 4);
   const uint32_t bar0 = smem_u32(smem + L::kOffBar);
   auto bar = [&](int i) -> uint32_t { return bar0 + 8u * (uint32_t)i; };
   const uint32_t q_base = smem_u32(smem + L::kOffQ);
   const uint32_t k_base = smem_u32(smem + L::kOffK);
   const uint32_t v_base = smem_u32(smem + L::kOffV);
   const uint32_t p_base = smem_u32(smem + L::kOffP);
+  const float NEG_INF = __int_as_float(0xff800000);
 
-  // ---- shape checks; every exit here is uniform over the cluster
+  // ---- the tree's extent (global reads in flight while the barriers are set up)
   const int off = a.node_off[b];
   const int n = a.node_off[b + 1] - off;
   const int P = a.prefix_len[b];
-  if (n < 1 || n > 256 || P < 0 || P + n > a.S_max || off < 0 || off + n > a.n_total) {
-    if (split == 0 && tid == 0 && blockIdx.y == 0) raise_status(a.status, kStTree);
-    return;
-  }
-  if (r0 >= G * n) return;
-  int bad = 0;
-  for (int v = tid; v < n; v += kThreads) {
-    const int p = a.parent[off + v];
-    par_s[v] = p;
-    bad |= (v == 0) ? (p != -1) : (p < 0 || p >= v);
-  }
-  if (__syncthreads_or(bad)) {
-    if (split == 0 && tid == 0 && blockIdx.y == 0) raise_status(a.status, kStTree);
-    return;
-  }
 
-  // ---- ancestor bitmasks of the nodes of this tile (row kBM stays zero)
-  const int u_base = r0 / G;
-  const int tile_nodes = min(kBM / G, n - u_base);
-  for (int i = tid; i < (kBM + 1) * kAncWords; i += kThreads) anc_s[i] = 0u;
-  __syncthreads();
-  for (int t = tid; t < tile_nodes; t += kThreads) {
-    uint32_t* w = anc_s + t * kAncWords;
-    for (int v = u_base + t; v >= 0; v = par_s[v]) w[v >> 5] |= 1u << (v & 31);
-  }
-
-  // ---- barriers and TMEM (S: columns [0,128), O: columns [128, 128 + D))
+  // ---- barriers; the first K/V copies go out before any global read returns
+  const int kv_row0 = (b * a.Hkv + h) * a.S_max;
+  auto load_kv = [&](int it) {  // it-th tile of this split = tile split + it * S_kv
+    const int st = it & 1;
+    mbar_arrive_expect_tx(bar(BAR_KV_FULL + st), 2 * L::kKVBytes);
+    const int y = kv_row0 + (split + it * S_kv) * kBN;
+#pragma unroll
+    for (int c = 0; c < D / 64; ++c) {
+      tma_load_2d(k_base + st * L::kKVBytes + c * kRegion, &tm_k, c * 64, y, bar(BAR_KV_FULL + st));
+      tma_load_2d(v_base + st * L::kKVBytes + c * kRegion, &tm_v, c * 64, y, bar(BAR_KV_FULL + st));
+    }
+  };
+  // Early copies are issued only for boxes that start inside the tensors (a
+  // box past the last row is never requested), and every issued copy is
+  // awaited before the buffers are reused or the CTA exits.
+  const int kv_rows = a.B * a.Hkv * a.S_max;
+  bool kv_early[kStages];
+#pragma unroll
+  for (int s = 0; s < kStages; ++s) kv_early[s] = kv_row0 + (split + s * S_kv) * kBN < kv_rows;
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(bar(BAR_KV_FULL + s), 1);
       mbar_init(bar(BAR_KV_EMPTY + s), 1);
+      mbar_init(bar(BAR_S_FULL + s), 1);
     }
     mbar_init(bar(BAR_Q_FULL), 1);
-    mbar_init(bar(BAR_S_FULL), 1);
-    mbar_init(bar(BAR_P_FULL), 128);
+    mbar_init(bar(BAR_P_FULL), kSoftmaxThreads);
     mbar_init(bar(BAR_O_DONE), 1);
     fence_mbar_init();
+    *bad_flag = 0;
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
+    tma_prefetch_desc(&tm_q);
+#pragma unroll
+    for (int s = 0; s < kStages; ++s)
+      if (kv_early[s]) load_kv(s);  // used when this split has that many tiles
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), 256);
+    tmem_alloc(smem_u32(tmem_slot), 512);  // S buffers: [0,128) [128,256); O: [256, 256 + D)
     tmem_relinquish();
+  }
+
+  // ---- shape checks (uniform over the cluster)
+  const bool bad_shape = (n < 1 || n > 256 || P < 0 || P + n > a.S_max || off < 0 ||
+                          off + n > a.n_total);
+  const bool skip = bad_shape || r0 >= G * n;
+  const int Lk = P + n;
+  const int T = (Lk + kBN - 1) / kBN;
+  const int nt = skip ? 0 : (split < T ? (T - split + S_kv - 1) / S_kv : 0);
+  const int u_base = r0 / G;
+  if (tid == 0 && nt > 0) {
+    mbar_arrive_expect_tx(bar(BAR_Q_FULL), L::kQBytes);
+#pragma unroll
+    for (int c = 0; c < D / 64; ++c)
+      tma_load_3d(q_base + c * kRegion, &tm_q, c * 64, h * G, off + u_base, bar(BAR_Q_FULL));
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tmem_S = tmem;
-  const uint32_t tmem_O = tmem + 128u;
-
-  // ---- this split's KV tiles
-  const int Lk = P + n;
-  const int T = (Lk + kBN - 1) / kBN;
-  const int t0 = (int)((long long)split * T / S_kv);
-  const int t1 = (int)((long long)(split + 1) * T / S_kv);
-  const int nt = t1 - t0;
-  const int kv_row0 = (b * a.Hkv + h) * a.S_max;
+  if (skip) {
+    // nothing to compute (uniform over the cluster): let the early copies land, leave
+    if (tid == 0) {
+      bool ok = true;
+      for (int s = 0; s < kStages; ++s)
+        if (kv_early[s]) ok = mbar_wait(bar(BAR_KV_FULL + s), 0) && ok;
+      if (!ok) raise_status(a.status, kStTimeout);
+      if (bad_shape && split == 0 && blockIdx.y == 0) raise_status(a.status, kStTree);
+    }
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem, 512);
+    return;
+  }
 
   if (warp == 0) {
     // ------------------------------------------------ TMA producer
-    if (lane == 0 && nt > 0) {
-      tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
-      mbar_arrive_expect_tx(bar(BAR_Q_FULL), L::kQBytes);
-#pragma unroll
-      for (int c = 0; c < D / 64; ++c)
-        tma_load_3d(q_base + c * kRegion, &tm_q, c * 64, h * G, off + u_base, bar(BAR_Q_FULL));
-      for (int it = 0; it < nt; ++it) {
+    if (lane == 0) {
+      // real tiles always lie inside the tensors, so an early stage was issued
+      // for each of the first min(nt, kStages) tiles
+      for (int it = kStages; it < nt; ++it) {
         const int st = it & 1;
-        if (it >= kStages && !mbar_wait(bar(BAR_KV_EMPTY + st), ((it >> 1) - 1) & 1)) {
+        if (!mbar_wait(bar(BAR_KV_EMPTY + st), ((it >> 1) - 1) & 1)) {
           raise_status(a.status, kStTimeout);
           break;
         }
-        mbar_arrive_expect_tx(bar(BAR_KV_FULL + st), 2 * L::kKVBytes);
-        const int y = kv_row0 + (t0 + it) * kBN;
-#pragma unroll
-        for (int c = 0; c < D / 64; ++c) {
-          tma_load_2d(k_base + st * L::kKVBytes + c * kRegion, &tm_k, c * 64, y,
-                      bar(BAR_KV_FULL + st));
-          tma_load_2d(v_base + st * L::kKVBytes + c * kRegion, &tm_v, c * 64, y,
-                      bar(BAR_KV_FULL + st));
-        }
+        load_kv(it);
       }
     }
     __syncwarp();
@@ -223,29 +247,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && nt > 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kBN, false);
       constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, true);
+      const uint32_t tmem_O = tmem + 256u;
       bool ok = mbar_wait(bar(BAR_Q_FULL), 0);
       for (int it = 0; ok && it <= nt; ++it) {
         if (it < nt) {
+          // S buffer it&1 was last read by the softmax of tile it-2, whose
+          // P_FULL phase was awaited before PV(it-2) was issued
           const int st = it & 1;
           ok = mbar_wait(bar(BAR_KV_FULL + st), (it >> 1) & 1);
-          if (ok && it > 0) ok = mbar_wait(bar(BAR_P_FULL), (it - 1) & 1);
           if (!ok) break;
           tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint32_t qa = q_base + (kk >> 2) * kRegion + (kk & 3) * 32;
             const uint32_t ka = k_base + st * L::kKVBytes + (kk >> 2) * kRegion + (kk & 3) * 32;
-            tc_mma_f16(tmem_S, smem_desc_sw128(qa, 16, 1024), smem_desc_sw128(ka, 16, 1024), kIdS,
-                       kk > 0 ? 1u : 0u);
+            tc_mma_f16(tmem + (uint32_t)(st * 128), smem_desc_sw128(qa, 16, 1024),
+                       smem_desc_sw128(ka, 16, 1024), kIdS, kk > 0 ? 1u : 0u);
           }
-          tc_commit(bar(BAR_S_FULL));
-        } else {
-          ok = mbar_wait(bar(BAR_P_FULL), (it - 1) & 1);
-          if (!ok) break;
-          tc_fence_after();
+          tc_commit(bar(BAR_S_FULL + st));
         }
         if (it > 0) {
           const int jt = it - 1, sp = jt & 1;
+          ok = mbar_wait(bar(BAR_P_FULL), jt & 1);
+          if (!ok) break;
+          tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < kBN / 16; ++kk) {
             const uint32_t pa = p_base + (kk >> 2) * kRegion + (kk & 3) * 32;
@@ -260,98 +285,130 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) raise_status(a.status, kStTimeout);
     }
     __syncwarp();
-  } else {
-    // ------------------------------------------------ softmax warps
-    const int q4 = warp & 3;              // TMEM lane quarter of this warp
-    const int r = q4 * 32 + lane;         // tile row = TMEM lane
-    const int rg = r0 + r;
-    const int u = rg / G;
+  }
+
+  // ------------------------------------------------ softmax warps
+  const int sidx = tid - 64;           // 0..255 for softmax threads
+  const int q4 = warp & 3;             // TMEM lane quarter of this warp
+  const int half = sidx >> 7;          // key / O column half
+  const int r = q4 * 32 + lane;        // tile row = TMEM lane
+  const float sl2 = a.scale_log2;      // softmax scale * log2(e): scores in base 2
+  if (warp >= 2) {
+    // parent array, validation and ancestor bitmasks, while the first
+    // copies and products are in flight (row kBM stays zero)
+    int bad = 0;
+    for (int v = sidx; v < n; v += kSoftmaxThreads) {
+      const int p = a.parent[off + v];
+      par_s[v] = p;
+      bad |= (v == 0) ? (p != -1) : (p < 0 || p >= v);
+    }
+    for (int i = sidx; i < (kBM + 1) * kAncWords; i += kSoftmaxThreads) anc_s[i] = 0u;
+    if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(bad_flag, 1);
+    softmax_bar();
+    if (*bad_flag == 0) {
+      const int tile_nodes = min(kBM / G, n - u_base);
+      for (int t = sidx; t < tile_nodes; t += kSoftmaxThreads) {
+        uint32_t* w = anc_s + t * kAncWords;
+        for (int v = u_base + t; v >= 0; v = par_s[v]) w[v >> 5] |= 1u << (v & 31);
+      }
+    } else if (sidx == 0 && split == 0) {
+      // a malformed tree keeps every tree slot masked; its outputs are undefined
+      raise_status(a.status, kStTree);
+    }
+    softmax_bar();
+
+    const int u = (r0 + r) / G;
     const uint32_t* anc = anc_s + (u < n ? (u - u_base) : kBM) * kAncWords;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
-    const float sl2 = a.scale_log2;
-    const float NEG_INF = __int_as_float(0xff800000);
-    float m_run = NEG_INF, l_run = 0.f;
+    const uint32_t tmem_O = tmem + 256u;
+    float m_run = NEG_INF, l_run = 0.f;  // m_run in raw score units
+    // Every softmax warp runs the same number of iterations and meets the
+    // named barrier in each one, also after a timed-out wait (then it only
+    // skips the work), so no warp is ever left waiting at that barrier.
     bool ok = true;
     for (int it = 0; it < nt; ++it) {
       const int st = it & 1;
-      const int key0 = (t0 + it) * kBN;
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_S_FULL), it & 1));
-      if (!ok) break;
-      tc_fence_after();
-      float s[kBN];
-#pragma unroll
-      for (int c = 0; c < kBN / 32; ++c)
-        tmem_ld32f(tmem_S + lane_off + c * 32, *reinterpret_cast<float(*)[32]>(&s[c * 32]));
-      tc_wait_ld();
+      const int tile_key0 = (split + it * S_kv) * kBN;
+      const int key0 = tile_key0 + half * 64;  // first key of this thread's columns
+      float s[64];
       float mx = NEG_INF;
-      if (key0 + kBN <= P) {
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_S_FULL + st), (it >> 1) & 1));
+      if (ok) {
+        tc_fence_after();
+        const uint32_t ts = tmem + (uint32_t)(st * 128) + lane_off + half * 64;
+        tmem_ld32f(ts, *reinterpret_cast<float(*)[32]>(&s[0]));
+        tmem_ld32f(ts + 32, *reinterpret_cast<float(*)[32]>(&s[32]));
+        tc_wait_ld();
+        if (key0 + 64 <= P) {
 #pragma unroll
-        for (int c = 0; c < kBN; ++c) {
-          s[c] *= sl2;
-          mx = fmaxf(mx, s[c]);
-        }
-      } else {
-        uint32_t mw[kBN / 32];
+          for (int c = 0; c < 64; ++c) mx = fmaxf(mx, s[c]);
+        } else {
+          const uint32_t mw0 = mask_word(anc, key0 - P);
+          const uint32_t mw1 = mask_word(anc, key0 + 32 - P);
 #pragma unroll
-        for (int w = 0; w < kBN / 32; ++w) mw[w] = mask_word(anc, key0 + 32 * w - P);
-#pragma unroll
-        for (int c = 0; c < kBN; ++c) {
-          const bool vis = (mw[c >> 5] >> (c & 31)) & 1u;
-          s[c] = vis ? s[c] * sl2 : NEG_INF;
-          mx = fmaxf(mx, s[c]);
+          for (int c = 0; c < 64; ++c) {
+            const bool vis = (((c < 32) ? mw0 : mw1) >> (c & 31)) & 1u;
+            s[c] = vis ? s[c] : NEG_INF;
+            mx = fmaxf(mx, s[c]);
+          }
         }
       }
-      const float m_new = fmaxf(m_run, mx);
+      // row max over both halves (double-buffered by tile parity)
+      float* rm = red_max + st * 2 * kBM;
+      rm[half * kBM + r] = mx;
+      softmax_bar();
+      if (!ok) continue;
+      const float m_new = fmaxf(m_run, fmaxf(rm[r], rm[kBM + r]));
       const float m_use = (m_new == NEG_INF) ? 0.f : m_new;
-      const float corr = ex2(m_run - m_use);
-      float rs = 0.f;
+      const float nb = -m_use * sl2;
+      const float corr = ex2(fmaf(m_run, sl2, nb));
+      float rs0 = 0.f, rs1 = 0.f;
 #pragma unroll
-      for (int c = 0; c < kBN; ++c) {
-        s[c] = ex2(s[c] - m_use);
-        rs += s[c];
+      for (int c = 0; c < 64; c += 2) {
+        s[c] = ex2(fmaf(s[c], sl2, nb));
+        s[c + 1] = ex2(fmaf(s[c + 1], sl2, nb));
+        rs0 += s[c];
+        rs1 += s[c + 1];
       }
-      l_run = l_run * corr + rs;
+      l_run = l_run * corr + (rs0 + rs1);
       if (it > 0) {
         // PV(it-1) must finish before O is rescaled and P is overwritten
         ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_O_DONE), (it - 1) & 1));
-        if (!ok) break;
+        if (!ok) continue;
         tc_fence_after();
         if (__any_sync(0xffffffffu, m_new > m_run)) {
 #pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
+          for (int c = 0; c < DH / 32; ++c) {
             uint32_t o[32];
-            tmem_ld32(tmem_O + lane_off + c * 32, o);
+            tmem_ld32(tmem_O + lane_off + half * DH + c * 32, o);
             tc_wait_ld();
 #pragma unroll
             for (int q = 0; q < 32; ++q) o[q] = __float_as_uint(__uint_as_float(o[q]) * corr);
-            tmem_st32(tmem_O + lane_off + c * 32, o);
+            tmem_st32(tmem_O + lane_off + half * DH + c * 32, o);
           }
           tc_wait_st();
         }
       }
-      if (key0 + kBN > Lk) {
+      if (tile_key0 + kBN > Lk) {
         // last tile of the sequence: V rows past the end may hold anything;
         // zero them so that 0-weight rows contribute exactly 0
         ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_KV_FULL + st), (it >> 1) & 1));
-        if (!ok) break;
-        if (key0 + r >= Lk) {
+        if (!ok) continue;
+        if (tile_key0 + r >= Lk && half < D / 64) {
 #pragma unroll
-          for (int c = 0; c < D / 64; ++c)
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-              st_shared_v4(v_base + st * L::kKVBytes + c * kRegion + r * 128 + q * 16,
-                           make_uint4(0u, 0u, 0u, 0u));
+          for (int q = 0; q < 8; ++q)
+            st_shared_v4(v_base + st * L::kKVBytes + half * kRegion + r * 128 + q * 16,
+                         make_uint4(0u, 0u, 0u, 0u));
         }
       }
-      // P row -> shared memory, bf16, 128-byte swizzled K-major operand layout
+      // this thread's 64 P columns -> region `half`, bf16, 128-byte swizzle
 #pragma unroll
-      for (int ch = 0; ch < kBN / 8; ++ch) {
+      for (int ch = 0; ch < 8; ++ch) {
         const uint4 w = make_uint4(pack_bf16(s[ch * 8 + 0], s[ch * 8 + 1]),
                                    pack_bf16(s[ch * 8 + 2], s[ch * 8 + 3]),
                                    pack_bf16(s[ch * 8 + 4], s[ch * 8 + 5]),
                                    pack_bf16(s[ch * 8 + 6], s[ch * 8 + 7]));
-        const int region = ch >> 3, chunk = ch & 7;
-        st_shared_v4(p_base + region * kRegion + r * 128 + ((chunk ^ (r & 7)) << 4), w);
+        st_shared_v4(p_base + half * kRegion + r * 128 + ((ch ^ (r & 7)) << 4), w);
       }
       fence_proxy_async_smem();
       tc_fence_before();
@@ -362,76 +419,142 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_O_DONE), (nt - 1) & 1));
       if (ok) tc_fence_after();
     }
-    float* ost = reinterpret_cast<float*>(smem + L::kOffO) + r * L::kOStride;
-    if (ok && nt > 0) {
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
-        uint32_t o[32];
-        tmem_ld32(tmem_O + lane_off + c * 32, o);
-        tc_wait_ld();
-#pragma unroll
-        for (int q = 0; q < 32; q += 4)
-          *reinterpret_cast<float4*>(ost + c * 32 + q) =
-              make_float4(__uint_as_float(o[q]), __uint_as_float(o[q + 1]),
-                          __uint_as_float(o[q + 2]), __uint_as_float(o[q + 3]));
-      }
-    } else {
-      for (int c = 0; c < D; c += 4) *reinterpret_cast<float4*>(ost + c) = make_float4(0, 0, 0, 0);
-      m_run = NEG_INF;
-      l_run = 0.f;
-      if (!ok && lane == 0) raise_status(a.status, kStTimeout);
-    }
-    m_s[r] = m_run;
-    l_s[r] = l_run;
-  }
+    // early K/V copies this split did not use land in the buffers the
+    // staging below reuses: wait for them first
+    for (int it = nt; it < kStages; ++it)
+      if (kv_early[it] && !mbar_wait(bar(BAR_KV_FULL + it), 0)) ok = false;
+    ok = __all_sync(0xffffffffu, ok);
+    if (!ok && lane == 0) raise_status(a.status, kStTimeout);
+    // row sum over both halves; every MMA of the CTA is done past this barrier
+    red_l[half * kBM + r] = l_run;
+    softmax_bar();
+    const float l_tot = red_l[r] + red_l[kBM + r];
+    const bool live = ok && nt > 0 && m_run != NEG_INF;
 
-  // ---- combine the S_kv partials of each row over DSMEM
-  tc_fence_before();
-  cluster.sync();
-  if (warp >= 2) {
-    const int st = tid - 64;
-    const int rpc = kBM / S_kv;
-    const int rbeg = split * rpc;
-    constexpr int C4 = D / 4;
-    const float NEG_INF = __int_as_float(0xff800000);
-    for (int item = st; item < rpc * C4; item += 128) {
-      const int rr = rbeg + item / C4, c4 = item % C4;
-      const int rg = r0 + rr;
+    if (S_kv == 1) {
+      // ---- single split: normalise this row's O columns and write them
+      const int rg = r0 + r;
       const int uu = rg / G, g = rg % G;
-      if (uu >= n) continue;
-      float M = NEG_INF;
-      for (int s = 0; s < S_kv; ++s) M = fmaxf(M, cluster.map_shared_rank(m_s, s)[rr]);
-      float Ls = 0.f;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (M != NEG_INF) {
-        for (int s = 0; s < S_kv; ++s) {
-          const float ms = cluster.map_shared_rank(m_s, s)[rr];
-          if (ms == NEG_INF) continue;
-          const float w = ex2(ms - M);
-          Ls += w * cluster.map_shared_rank(l_s, s)[rr];
-          const float* po = reinterpret_cast<const float*>(smem + L::kOffO);
-          const float4 o = *reinterpret_cast<const float4*>(
-              cluster.map_shared_rank(po, s) + rr * L::kOStride + c4 * 4);
-          acc.x += w * o.x;
-          acc.y += w * o.y;
-          acc.z += w * o.z;
-          acc.w += w * o.w;
+      const float inv = (live && l_tot > 0.f) ? 1.f / l_tot : 0.f;
+      const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
+#pragma unroll
+      for (int c = 0; c < DH / 32; ++c) {
+        float o[32];
+        tmem_ld32f(tmem_O + lane_off + half * DH + c * 32, o);
+        tc_wait_ld();
+        if (uu < n) {
+          uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D +
+                                                half * DH + c * 32);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            dst[q] = make_uint4(pack_bf16(o[8 * q + 0] * inv, o[8 * q + 1] * inv),
+                                pack_bf16(o[8 * q + 2] * inv, o[8 * q + 3] * inv),
+                                pack_bf16(o[8 * q + 4] * inv, o[8 * q + 5] * inv),
+                                pack_bf16(o[8 * q + 6] * inv, o[8 * q + 7] * inv));
         }
       }
-      const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
-      const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
-      uint2 pk;
-      pk.x = pack_bf16(acc.x * inv, acc.y * inv);
-      pk.y = pack_bf16(acc.z * inv, acc.w * inv);
-      *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c4 * 4) = pk;
-      if (c4 == 0 && a.lse_out) a.lse_out[orow] = (M + log2f(Ls)) * kLn2;
+      if (half == 0 && uu < n && a.lse_out)
+        a.lse_out[orow] = live ? (m_run * sl2 + log2f(l_tot)) * kLn2 : NEG_INF;
+    } else {
+      // ---- stage this row's partial: [O (D fp32) | m (base 2) | l | pad]
+      float* row = stage_rows + r * L::kRowFloats;
+      // tcgen05.ld / wait::ld are warp-collective: the condition must be the
+      // same for the 32 lanes (ok and nt are); per-row liveness only selects
+      // what is stored
+      if (ok && nt > 0) {
+#pragma unroll
+        for (int c = 0; c < DH / 32; ++c) {
+          float o[32];
+          tmem_ld32f(tmem_O + lane_off + half * DH + c * 32, o);
+          tc_wait_ld();
+#pragma unroll
+          for (int q = 0; q < 32; q += 4)
+            *reinterpret_cast<float4*>(row + half * DH + c * 32 + q) =
+                live ? make_float4(o[q], o[q + 1], o[q + 2], o[q + 3])
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      } else {
+        for (int c = 0; c < DH; c += 4)
+          *reinterpret_cast<float4*>(row + half * DH + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+      if (half == 0) {
+        row[D] = live ? m_run * sl2 : NEG_INF;
+        row[D + 1] = live ? l_tot : 0.f;
+      }
     }
   }
-  cluster.sync();
+  tc_fence_before();
+  if (S_kv == 1) {
+    __syncthreads();  // TMEM reads are done
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc(tmem, 512);
+    }
+    return;
+  }
+
+  // ---- combine: each CTA pulls the S_kv partials of the rows it owns
+  cluster.sync();  // every CTA's partial rows are staged; its MMAs and TMEM use are over
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 256);
+    tmem_dealloc(tmem, 512);
   }
+  const int rpc = (kBM + S_kv - 1) / S_kv;  // tile rows owned by each CTA of the cluster
+  const int row_lo = split * rpc;
+  const int my_rows = max(0, min(kBM, row_lo + rpc) - row_lo);
+  constexpr int CG = D / 8;  // 8-column groups per row
+  for (int item = tid; item < my_rows * CG; item += kThreads) {
+    const int rr = row_lo + item / CG, c8 = item % CG;
+    const int rg = r0 + rr;
+    const int uu = rg / G, g = rg % G;
+    // issue every peer load before using any of them
+    float mv[kMaxSplits], lv[kMaxSplits];
+    float4 ov[kMaxSplits][2];
+#pragma unroll
+    for (int sp = 0; sp < kMaxSplits; ++sp) {
+      if (sp < S_kv) {
+        const float* src = cluster.map_shared_rank(stage_rows, sp) + rr * L::kRowFloats;
+        mv[sp] = src[D];
+        lv[sp] = src[D + 1];
+        ov[sp][0] = *reinterpret_cast<const float4*>(src + c8 * 8);
+        ov[sp][1] = *reinterpret_cast<const float4*>(src + c8 * 8 + 4);
+      }
+    }
+    if (uu >= n) continue;
+    float M = NEG_INF;
+#pragma unroll
+    for (int sp = 0; sp < kMaxSplits; ++sp)
+      if (sp < S_kv) M = fmaxf(M, mv[sp]);
+    float Ls = 0.f;
+    float acc[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+#pragma unroll
+    for (int sp = 0; sp < kMaxSplits; ++sp) {
+      if (sp < S_kv) {
+        const float w = (mv[sp] == NEG_INF) ? 0.f : ex2(mv[sp] - M);
+        Ls += w * lv[sp];
+        acc[0] += w * ov[sp][0].x;
+        acc[1] += w * ov[sp][0].y;
+        acc[2] += w * ov[sp][0].z;
+        acc[3] += w * ov[sp][0].w;
+        acc[4] += w * ov[sp][1].x;
+        acc[5] += w * ov[sp][1].y;
+        acc[6] += w * ov[sp][1].z;
+        acc[7] += w * ov[sp][1].w;
+      }
+    }
+    const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
+    const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
+    uint4 pk;
+    pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+    pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+    pk.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+    pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+    *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c8 * 8) = pk;
+    if (c8 == 0 && a.lse_out) a.lse_out[orow] = (M == NEG_INF) ? M : (M + log2f(Ls)) * kLn2;
+  }
+  cluster.sync();  // peers may still be reading this CTA's staged rows until here
 }
 
 template <int D>
@@ -458,27 +581,67 @@ cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtenso
   return cudaLaunchKernelEx(&cfg, kern, tq, tk, tv, a);
 }
 
+// clusters of `splits` CTAs of this kernel that can be resident at once
+template <int D>
+int max_active_clusters_d(int splits) {
+  using L = Layout<D>;
+  auto kern = tree_attn_kernel<D>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc) !=
+      cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(splits, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = L::kAlloc;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
 }  // namespace
 
-// KV splits per work item: the power of two in {1, 2, 4, 8} whose grid fills
-// the SMs best (one CTA per SM), preferring fewer splits on near ties.
-int tree_attn_pick_splits(int B, int Hkv, int mtiles, int S_max, int num_sms) {
+// KV splits per work item.  Cost model: waves of resident clusters times the
+// per-CTA time, a fixed part plus one part per 128-key tile of its split.
+// The number of clusters that fit at once comes from the occupancy API
+// (cached per device, head size and split count).
+int tree_attn_pick_splits(int D, int B, int Hkv, int mtiles, int S_max, int num_sms) {
+  static int cache[64][2][kMaxSplits + 1] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
+  const int di = D == 64 ? 0 : 1;
   const long long units = (long long)B * Hkv * mtiles;
-  const int max_tiles = (S_max + kBN - 1) / kBN;
+  const int tiles = (S_max + kBN - 1) / kBN;
+  const double kFixed = 5.0, kCombine = 1.0, kPerTile = 0.9;  // microseconds, measured scale
   int best = 1;
-  double best_eff = -1.0;
-  for (int s = 1; s <= 8; s *= 2) {
-    if (s > 1 && s > max_tiles) break;
-    const long long ctas = units * s;
-    const long long waves = (ctas + num_sms - 1) / num_sms;
-    const double eff = (double)ctas / (double)(waves * num_sms);
-    if (eff > best_eff + 0.03) {
-      best_eff = eff;
+  double best_cost = 1e30;
+  for (int s = 1; s <= kMaxSplits; ++s) {
+    if (s > 1 && s > tiles) break;
+    int& fit = cache[dev][di][s];
+    if (fit == 0) fit = di ? max_active_clusters_d<128>(s) : max_active_clusters_d<64>(s);
+    const int resident = fit > 0 ? fit : (s == 1 ? num_sms : num_sms / (2 * s));
+    if (resident <= 0) continue;
+    const long long waves = (units + resident - 1) / resident;
+    const double cost = (double)waves * (kFixed + (s > 1 ? kCombine : 0.0) +
+                                         kPerTile * (double)((tiles + s - 1) / s));
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
       best = s;
     }
   }
   return best;
 }
+
+
 
 cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                              const CUtensorMap& tm_v, const AttnArgs& a, int kv_splits,

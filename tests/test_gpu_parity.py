@@ -177,20 +177,27 @@ def test_expand_topk_ragged_vocab(dev, V, ld, dtype, k):
     _check_expand(got, ref)
 
 
-def test_expand_topk_ties_inf_and_row_idx(dev):
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_expand_topk_ties_inf_and_row_idx(dev, dtype):
+    # heavy ties overflow the candidate buffer and take the exact-key fallback
     rng = synth.make_rng(5)
-    V = 5000
+    V = 5000 if dtype == "f32" else 40000
     x = rng.integers(-1, 2, size=(6, V)).astype(np.float32)     # heavy ties
     x[2] = -np.inf                                              # all -inf row
     x[3, ::3] = -np.inf
     x[4] = 0.0
-    x[4, 4999] = 0.5
     x[5, :] = -0.0
     x[5, 17] = 0.0
+    x[4, V - 1] = 0.5
     ps = np.array([0, -1, -2, -3, -4, -5, -6, -7], np.float32)
     row_idx = np.array([5, 4, 3, 0, 1, 0, 2, 2], np.int32)
-    got = _run_expand(_dev.f32(x, dev), ps, 12, dev, row_idx=row_idx)
-    ref = O.expand_topk(x, ps, 12, row_idx=row_idx)
+    if dtype == "f32":
+        got = _run_expand(_dev.f32(x, dev), ps, 12, dev, row_idx=row_idx)
+        ref = O.expand_topk(x, ps, 12, row_idx=row_idx)
+    else:
+        bits = synth.f32_to_bf16_bits(x)
+        got = _run_expand(_dev.bf16(bits, dev), ps, 12, dev, row_idx=row_idx)
+        ref = O.expand_topk(bits, ps, 12, row_idx=row_idx, bf16=True)
     np.testing.assert_array_equal(got[0], ref[0])
     for g, r in zip(got[1:], ref[1:]):
         np.testing.assert_array_equal(np.isneginf(g), np.isneginf(r))
@@ -270,6 +277,23 @@ def test_accept_bit_exact(dev, name, bump):
     # the workspace is ready for a second call: same answer
     got2 = _run_accept(wl, dev, cap)
     for g, r in zip(got2[:3], ref):
+        np.testing.assert_array_equal(g, r)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_accept_tied_logits(dev, dtype):
+    # quantised target logits: every row's argmax is decided by the lowest-token rule
+    wl = synth.make_workload("llama3-8b-verify", seed=11, with_logits=False, with_strong=False)
+    rng = synth.make_rng(12)
+    V = 50000
+    x = rng.integers(-1, 2, size=(len(wl["parent"]), V)).astype(np.float32)
+    x[:, :3] = -1.0
+    wl["logits"] = x if dtype == "f32" else synth.f32_to_bf16_bits(x)
+    cap = _dev.max_nodes(wl)
+    got = _run_accept(wl, dev, cap)
+    ref = O.accept(wl["logits"], wl["token"], wl["parent"], wl["node_off"], cap,
+                   bf16=(dtype == "bf16"))
+    for g, r in zip(got[:3], ref):
         np.testing.assert_array_equal(g, r)
 
 
