@@ -132,7 +132,10 @@ def alloc_outputs(d, sh, dev):
         path=torch.empty(1, n, dtype=torch.int32, device=dev),
         alen=torch.empty(1, dtype=torch.int32, device=dev),
         bonus=torch.empty(1, dtype=torch.int32, device=dev),
-        ws=tg.accept_workspace(1, n, dev))
+        ws=tg.accept_workspace(1, n, dev),
+        attn_ws=torch.empty(max(16, tg.tree_attn_workspace_size(
+            1, n, d["q"].shape[1], d["k"].shape[1], d["q"].shape[2])), dtype=torch.uint8,
+            device=dev))
 
 
 def call(name, d, o, sh):
@@ -140,7 +143,7 @@ def call(name, d, o, sh):
     n = d["parent"].shape[0]
     if name == "tree_attn":
         tg.tree_attn(d["q"], d["k"], d["v"], d["prefix_len"], d["parent"], d["node_off"], n,
-                     out=o["o"])
+                     out=o["o"], ws=o["attn_ws"])
     elif name == "expand_topk":
         tg.expand_topk(d["logits"], d["parent_score"], sh["k"], out=(o["tok"], o["lp"], o["sc"]))
     elif name == "rescore_select":

@@ -76,6 +76,10 @@ typedef enum { TG_BF16 = 0, TG_F32 = 1 } tg_dtype;
  * D in {64, 128}; Hq % Hkv == 0, G = Hq / Hkv in {1, 2, 4, 8}.
  * scale    softmax scale; 0 selects D^-1/2.
  * out      bf16 [n_total, Hq, D];  lse_out fp32 [n_total, Hq] or NULL.
+ * ws       scratch of treegraft_tree_attn_workspace_size(B, max_nodes, Hq,
+ *          Hkv, D) bytes, 16-byte aligned: partial rows of the split-KV
+ *          combine (needs no initialisation).  Calls sharing one ws must not
+ *          overlap on the GPU.
  * Errors: TG_ERR_INVALID_ARG (null pointer, bad sizes, misaligned q/k/v),
  *   TG_ERR_UNSUPPORTED (D or G outside the list), TG_ERR_CUDA.  A malformed
  *   tree sets TG_ERR_DEVICE_TREE; its rows of `out` and `lse_out` are then
@@ -85,7 +89,13 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
                         const int32_t* prefix_len, const int32_t* parent,
                         const int32_t* node_off, int B, int max_nodes, int n_total,
                         int Hq, int Hkv, int D, int S_max, float scale,
-                        void* out, float* lse_out, void* stream);
+                        void* out, float* lse_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * treegraft_tree_attn_workspace_size - bytes of scratch treegraft_tree_attn
+ * needs for these sizes (0 for invalid sizes).  Depends on no device state.
+ */
+size_t treegraft_tree_attn_workspace_size(int B, int max_nodes, int Hq, int Hkv, int D);
 
 /*
  * treegraft_expand_topk - per-node log-softmax, top-k children, path scores.

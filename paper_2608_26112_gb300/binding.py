@@ -36,7 +36,9 @@ _c_int, _c_i64, _c_f32, _c_vp, _c_size = (ctypes.c_int, ctypes.c_int64, ctypes.c
 
 _SIGNATURES = {
     "treegraft_tree_attn": [_c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_int, _c_int, _c_int,
-                            _c_int, _c_int, _c_int, _c_int, _c_f32, _c_vp, _c_vp, _c_vp],
+                            _c_int, _c_int, _c_int, _c_int, _c_f32, _c_vp, _c_vp, _c_vp, _c_size,
+                            _c_vp],
+    "treegraft_tree_attn_workspace_size": [_c_int, _c_int, _c_int, _c_int, _c_int],
     "treegraft_expand_topk": [_c_vp, _c_int, _c_int, _c_int, _c_i64, _c_int, _c_vp, _c_vp,
                               _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp],
     "treegraft_rescore_select": [_c_vp, _c_vp, _c_int, _c_i64, _c_vp, _c_vp, _c_vp, _c_vp,
@@ -51,6 +53,7 @@ _SIGNATURES = {
     "treegraft_status_string": [_c_int],
 }
 _RESTYPES = {"treegraft_accept_workspace_size": _c_size,
+             "treegraft_tree_attn_workspace_size": _c_size,
              "treegraft_status_string": ctypes.c_char_p}
 
 
@@ -105,11 +108,16 @@ def _logit_dtype(t):
     raise TypeError("logits must be bfloat16 or float32")
 
 
+def tree_attn_workspace_size(B, max_nodes, Hq, Hkv, D) -> int:
+    return int(lib().treegraft_tree_attn_workspace_size(B, int(max_nodes), Hq, Hkv, D))
+
+
 def tree_attn(q, k_cache, v_cache, prefix_len, parent, node_off, max_nodes, *, scale=0.0,
-              out=None, lse_out=None, stream=None):
+              out=None, lse_out=None, ws=None, stream=None):
     """Ancestor-masked GQA tree attention.  q [n_total, Hq, D] bf16,
     k_cache / v_cache [B, Hkv, S_max, D] bf16, prefix_len [B] int32,
-    parent [n_total] int32 (local ids), node_off [B+1] int32.
+    parent [n_total] int32 (local ids), node_off [B+1] int32.  ws: uint8
+    scratch of tree_attn_workspace_size() bytes (allocated here if None).
     Returns (out [n_total, Hq, D] bf16, lse_out or None)."""
     _need(q, torch.bfloat16, "q")
     _need(k_cache, torch.bfloat16, "k_cache")
@@ -125,10 +133,14 @@ def tree_attn(q, k_cache, v_cache, prefix_len, parent, node_off, max_nodes, *, s
     _need(out, torch.bfloat16, "out")
     if lse_out is not None:
         _need(lse_out, torch.float32, "lse_out")
+    if ws is None:
+        ws = torch.empty(max(16, tree_attn_workspace_size(B, max_nodes, Hq, Hkv, D)),
+                         dtype=torch.uint8, device=q.device)
+    _need(ws, torch.uint8, "ws")
     st = lib().treegraft_tree_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(prefix_len),
                                    _ptr(parent), _ptr(node_off), B, int(max_nodes), n_total, Hq,
                                    Hkv, D, S_max, float(scale), _ptr(out), _ptr(lse_out),
-                                   _stream(stream))
+                                   _ptr(ws), ws.numel(), _stream(stream))
     _check("treegraft_tree_attn", st)
     return out, lse_out
 

@@ -96,10 +96,17 @@ using namespace tg;
 
 extern "C" {
 
+size_t treegraft_tree_attn_workspace_size(int B, int max_nodes, int Hq, int Hkv, int D) {
+  if (B < 1 || max_nodes < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || (D != 64 && D != 128)) return 0;
+  const int mtiles = ((Hq / Hkv) * max_nodes + 127) / 128;
+  return tree_attn_ws_bytes(D, B, Hkv, mtiles, 8);
+}
+
 int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
                         const int32_t* prefix_len, const int32_t* parent, const int32_t* node_off,
                         int B, int max_nodes, int n_total, int Hq, int Hkv, int D, int S_max,
-                        float scale, void* out, float* lse_out, void* stream) {
+                        float scale, void* out, float* lse_out, void* ws, size_t ws_bytes,
+                        void* stream) {
   if (!q || !k_cache || !v_cache || !prefix_len || !parent || !node_off || !out)
     return TG_ERR_INVALID_ARG;
   if (B < 1 || max_nodes < 1 || max_nodes > TG_MAX_TREE_NODES || n_total < 1 || Hq < 1 ||
@@ -149,6 +156,9 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
   a.status = st;
   const int mtiles = (G * max_nodes + 127) / 128;
   const int splits = tree_attn_pick_splits(D, B, Hkv, mtiles, S_max, device_sm_count());
+  const size_t need = tree_attn_ws_bytes(D, B, Hkv, mtiles, splits);
+  if (need > 0 && (ws == nullptr || ws_bytes < need || !aligned16(ws))) return TG_ERR_INVALID_ARG;
+  a.ws = ws;
   return launch_tree_attn(tq, tk, tv, a, splits, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? TG_OK
              : TG_ERR_CUDA;

@@ -16,6 +16,7 @@ struct AttnArgs {
   float scale_log2;  // softmax scale * log2(e)
   void* out;
   float* lse_out;
+  void* ws;  // split-combine partial rows (tree_attn_ws_bytes)
   int* status;
 };
 // tmaps: q [D, Hq, n_total], k and v [D, B*Hkv*S_max] (innermost first)
@@ -23,6 +24,7 @@ cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                              const CUtensorMap& tm_v, const AttnArgs& a, int kv_splits,
                              cudaStream_t s);
 int tree_attn_pick_splits(int D, int B, int Hkv, int mtiles, int S_max, int num_sms);
+size_t tree_attn_ws_bytes(int D, int B, int Hkv, int mtiles, int splits);
 
 struct TopkArgs {
   const void* logits;

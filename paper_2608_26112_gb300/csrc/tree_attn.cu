@@ -25,10 +25,10 @@
 //               P as bf16 into the swizzled operand layout, and rescale O in
 //               TMEM when the running max grows.
 // Split combine: each CTA stages its partial rows (O, max, sum) in shared
-// memory; between two cluster barriers every CTA reads the S_kv partials of
-// the rows it owns from its peers' shared memory (DSMEM) and writes the
-// normalised rows.  With a single split the rows are normalised and written
-// straight from TMEM.  Every mbarrier wait is bounded.
+// memory, copies them with coalesced stores into the caller's workspace (L2
+// resident), and after one cluster barrier reduces the S_kv partials of the
+// rows it owns, read back from L2.  With a single split the rows are
+// normalised and written straight from TMEM.  Every mbarrier wait is bounded.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -75,13 +75,14 @@ struct Layout {
   // Partial rows of the combine, written once every MMA of the CTA is done,
   // over the Q / K tiles: a row is [O (D fp32) | m (base 2) | l | 2 pad].
   static constexpr int kRowFloats = D + 4;
+  static constexpr int kSlabBytes = kBM * kRowFloats * 4;            // one CTA's partial rows
   static constexpr int kOffStage = 0;
-  static_assert(kOffStage + kBM * kRowFloats * 4 <= kTileEnd, "staging fits the tiles");
+  static_assert(kOffStage + kSlabBytes <= kTileEnd, "staging fits the tiles");
   static_assert(kAlloc <= 227 * 1024, "shared memory budget");
   static_assert(kOffQ % 1024 == 0 && kOffK % 1024 == 0 && kOffV % 1024 == 0 && kOffP % 1024 == 0,
                 "128-byte-swizzled operand tiles need 1024-byte alignment");
   static_assert(kOffBar % 8 == 0 && kOffMisc % 16 == 0, "mbarrier / scalar alignment");
-  static_assert((kRowFloats * 4) % 16 == 0, "float4 staging rows");
+  static_assert((kRowFloats * 4) % 16 == 0 && kSlabBytes % 16 == 0, "float4 staging rows");
 };
 
 // 32 mask bits of one node for tree slots [b0, b0 + 32): slot < 0 is the
@@ -172,6 +173,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   bool kv_early[kStages];
 #pragma unroll
   for (int s = 0; s < kStages; ++s) kv_early[s] = kv_row0 + (split + s * S_kv) * kBN < kv_rows;
+  auto load_q = [&](int node0) {
+    mbar_arrive_expect_tx(bar(BAR_Q_FULL), L::kQBytes);
+#pragma unroll
+    for (int c = 0; c < D / 64; ++c)
+      tma_load_3d(q_base + c * kRegion, &tm_q, c * 64, h * G, node0, bar(BAR_Q_FULL));
+  };
+  // tree 0 starts at node 0 (node_off[0] = 0), so its q tile is known up front
+  const bool q_early = (b == 0) && (r0 / G < a.n_total);
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(bar(BAR_KV_FULL + s), 1);
@@ -186,6 +195,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tm_k);
     tma_prefetch_desc(&tm_v);
     tma_prefetch_desc(&tm_q);
+    if (q_early) load_q(r0 / G);
 #pragma unroll
     for (int s = 0; s < kStages; ++s)
       if (kv_early[s]) load_kv(s);  // used when this split has that many tiles
@@ -197,18 +207,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---- shape checks (uniform over the cluster)
   const bool bad_shape = (n < 1 || n > 256 || P < 0 || P + n > a.S_max || off < 0 ||
-                          off + n > a.n_total);
+                          off + n > a.n_total || (b == 0 && off != 0));
   const bool skip = bad_shape || r0 >= G * n;
   const int Lk = P + n;
   const int T = (Lk + kBN - 1) / kBN;
   const int nt = skip ? 0 : (split < T ? (T - split + S_kv - 1) / S_kv : 0);
   const int u_base = r0 / G;
-  if (tid == 0 && nt > 0) {
-    mbar_arrive_expect_tx(bar(BAR_Q_FULL), L::kQBytes);
-#pragma unroll
-    for (int c = 0; c < D / 64; ++c)
-      tma_load_3d(q_base + c * kRegion, &tm_q, c * 64, h * G, off + u_base, bar(BAR_Q_FULL));
-  }
+  if (tid == 0 && !q_early && nt > 0) load_q(off + u_base);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -219,6 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int s = 0; s < kStages; ++s)
         if (kv_early[s]) ok = mbar_wait(bar(BAR_KV_FULL + s), 0) && ok;
+      if (q_early) ok = mbar_wait(bar(BAR_Q_FULL), 0) && ok;
       if (!ok) raise_status(a.status, kStTimeout);
       if (bad_shape && split == 0 && blockIdx.y == 0) raise_status(a.status, kStTree);
     }
@@ -419,10 +425,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_O_DONE), (nt - 1) & 1));
       if (ok) tc_fence_after();
     }
-    // early K/V copies this split did not use land in the buffers the
+    // speculative K/V copies this split did not use land in the buffers the
     // staging below reuses: wait for them first
     for (int it = nt; it < kStages; ++it)
       if (kv_early[it] && !mbar_wait(bar(BAR_KV_FULL + it), 0)) ok = false;
+    if (nt == 0 && q_early && !mbar_wait(bar(BAR_Q_FULL), 0)) ok = false;  // no MMA waited it
     ok = __all_sync(0xffffffffu, ok);
     if (!ok && lane == 0) raise_status(a.status, kStTimeout);
     // row sum over both halves; every MMA of the CTA is done past this barrier
@@ -493,12 +500,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
 
-  // ---- combine: each CTA pulls the S_kv partials of the rows it owns
-  cluster.sync();  // every CTA's partial rows are staged; its MMAs and TMEM use are over
+  // ---- combine through L2: publish this CTA's partial rows, then reduce the owned rows
+  __syncthreads();  // TMEM reads are done; the staged rows are complete
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
+  const size_t unit = (size_t)blockIdx.z * gridDim.y + blockIdx.y;
+  float* slabs = reinterpret_cast<float*>(a.ws) + unit * (size_t)S_kv * (L::kSlabBytes / 4);
+  {
+    float4* dst = reinterpret_cast<float4*>(slabs + (size_t)split * (L::kSlabBytes / 4));
+    const float4* src = reinterpret_cast<const float4*>(stage_rows);
+    for (int i = tid; i < L::kSlabBytes / 16; i += kThreads) __stcg(dst + i, src[i]);
+  }
+  __threadfence();
+  cluster.sync();  // every CTA of the cluster has published its rows
   const int rpc = (kBM + S_kv - 1) / S_kv;  // tile rows owned by each CTA of the cluster
   const int row_lo = split * rpc;
   const int my_rows = max(0, min(kBM, row_lo + rpc) - row_lo);
@@ -507,20 +523,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rr = row_lo + item / CG, c8 = item % CG;
     const int rg = r0 + rr;
     const int uu = rg / G, g = rg % G;
-    // issue every peer load before using any of them
+    if (uu >= n) continue;
+    // issue every load before using any of them
     float mv[kMaxSplits], lv[kMaxSplits];
     float4 ov[kMaxSplits][2];
 #pragma unroll
     for (int sp = 0; sp < kMaxSplits; ++sp) {
       if (sp < S_kv) {
-        const float* src = cluster.map_shared_rank(stage_rows, sp) + rr * L::kRowFloats;
-        mv[sp] = src[D];
-        lv[sp] = src[D + 1];
-        ov[sp][0] = *reinterpret_cast<const float4*>(src + c8 * 8);
-        ov[sp][1] = *reinterpret_cast<const float4*>(src + c8 * 8 + 4);
+        const float* src = slabs + (size_t)sp * (L::kSlabBytes / 4) + rr * L::kRowFloats;
+        mv[sp] = __ldcg(src + D);
+        lv[sp] = __ldcg(src + D + 1);
+        ov[sp][0] = __ldcg(reinterpret_cast<const float4*>(src + c8 * 8));
+        ov[sp][1] = __ldcg(reinterpret_cast<const float4*>(src + c8 * 8 + 4));
       }
     }
-    if (uu >= n) continue;
     float M = NEG_INF;
 #pragma unroll
     for (int sp = 0; sp < kMaxSplits; ++sp)
@@ -554,7 +570,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c8 * 8) = pk;
     if (c8 == 0 && a.lse_out) a.lse_out[orow] = (M == NEG_INF) ? M : (M + log2f(Ls)) * kLn2;
   }
-  cluster.sync();  // peers may still be reading this CTA's staged rows until here
 }
 
 template <int D>
@@ -642,6 +657,12 @@ int tree_attn_pick_splits(int D, int B, int Hkv, int mtiles, int S_max, int num_
 }
 
 
+
+size_t tree_attn_ws_bytes(int D, int B, int Hkv, int mtiles, int splits) {
+  if (splits <= 1) return 0;
+  const size_t slab = D == 64 ? (size_t)Layout<64>::kSlabBytes : (size_t)Layout<128>::kSlabBytes;
+  return (size_t)B * Hkv * mtiles * splits * slab;
+}
 
 cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                              const CUtensorMap& tm_v, const AttnArgs& a, int kv_splits,

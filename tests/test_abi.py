@@ -42,6 +42,12 @@ def test_status_strings(lib):
     assert b"invalid" in lib.treegraft_status_string(1)
 
 
+def test_tree_attn_workspace_size(lib):
+    # one fp32 slab of 128 rows x (D + 4) floats per (tree, kv-head, row tile, split), 8 splits
+    assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 128) == 1 * 8 * 2 * 8 * 128 * 132 * 4
+    assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 96) == 0
+
+
 def test_workspace_size(lib):
     assert lib.treegraft_accept_workspace_size(1, 60) >= 61 * 4
     assert lib.treegraft_accept_workspace_size(1, 60) % 256 == 0
@@ -55,23 +61,23 @@ def test_tree_attn_rejects_bad_args_on_host(lib):
     fake = ctypes.c_void_p(0x1000)
     # null pointer
     assert lib.treegraft_tree_attn(NULL, fake, fake, fake, fake, fake, 1, 16, 16, 8, 8, 64, 144,
-                                   0.0, fake, NULL, NULL) == 1
+                                   0.0, fake, NULL, NULL, 0, NULL) == 1
     # head_dim 96 unsupported, G = 3 unsupported, Hq % Hkv != 0 invalid
     assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 16, 16, 8, 8, 96, 144,
-                                   0.0, fake, NULL, NULL) == 2
+                                   0.0, fake, NULL, NULL, 0, NULL) == 2
     assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 16, 16, 12, 4, 64, 144,
-                                   0.0, fake, NULL, NULL) == 2
+                                   0.0, fake, NULL, NULL, 0, NULL) == 2
     assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 16, 16, 8, 3, 64, 144,
-                                   0.0, fake, NULL, NULL) == 1
+                                   0.0, fake, NULL, NULL, 0, NULL) == 1
     # more than 256 nodes per tree
     assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 300, 300, 8, 8, 64,
-                                   400, 0.0, fake, NULL, NULL) == 1
+                                   400, 0.0, fake, NULL, NULL, 0, NULL) == 1
     # misaligned q
     assert lib.treegraft_tree_attn(ctypes.c_void_p(0x1002), fake, fake, fake, fake, fake, 1, 16,
-                                   16, 8, 8, 64, 144, 0.0, fake, NULL, NULL) == 1
+                                   16, 8, 8, 64, 144, 0.0, fake, NULL, NULL, 0, NULL) == 1
     # negative scale
     assert lib.treegraft_tree_attn(fake, fake, fake, fake, fake, fake, 1, 16, 16, 8, 8, 64, 144,
-                                   -1.0, fake, NULL, NULL) == 1
+                                   -1.0, fake, NULL, NULL, 0, NULL) == 1
 
 
 def test_expand_topk_rejects_bad_args_on_host(lib):
