@@ -299,7 +299,8 @@ def run_cpu_oracle(steps, warmup, min_s, max_s):
 
 def traffic_record(kernel):
     """dram read+write bytes per launch from the committed ncu summary, or
-    None if the kernel's source changed since those counters were taken."""
+    None if any source the kernel is built from changed since those counters
+    were taken."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if not os.path.exists(path):
         return None
@@ -307,10 +308,15 @@ def traffic_record(kernel):
         rec = json.load(f).get(kernel)
     if not rec:
         return None
-    src = os.path.join(ROOT, "paper_2608_26112_gb300", "csrc", rec["source"])
-    with open(src, "rb") as f:
-        h = hashlib.sha256(f.read()).hexdigest()[:16]
-    return rec["bytes_per_launch"] if h == rec.get("source_sha256_16") else None
+    return rec["bytes_per_launch"] if sources_hash(rec["sources"]) == rec.get("sources_sha256_16") else None
+
+
+def sources_hash(names):
+    h = hashlib.sha256()
+    for name in names:
+        with open(os.path.join(ROOT, "paper_2608_26112_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 # --------------------------------------------------------------------------- arms
@@ -327,14 +333,28 @@ def dist_setup(args):
     return world, rank, local
 
 
+def rank_seed(seed, rank):
+    """Each rank draws its own sequences: the ranks share no input and the
+    step has no exchange between them."""
+    return seed + 1000 * rank
+
+
 def max_over_ranks(x, world):
+    """Slowest rank's time (the job's time): an all-reduce of one float on
+    the host side of the timing, never inside the timed step."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(world, steps, t_max):
+    """Whole-job steps/s: every rank runs `steps` steps of its own sequences."""
+    return world * steps / t_max
 
 
 def barrier(world):
@@ -342,7 +362,8 @@ def barrier(world):
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
-    torch.cuda.synchronize()
+    if torch.cuda.is_available():
+        torch.cuda.synchronize()
 
 
 def reference_arm(args):
@@ -382,7 +403,7 @@ def ours_arm(args):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     R = args.sets
-    sets, host = build_sets(R, args.seed + 1000 * rank, dev)
+    sets, host = build_sets(R, rank_seed(args.seed, rank), dev)
     sh = host[0]["shape"]
     outs = [alloc_outputs(d, sh, dev) for d in sets]
     stream = torch.cuda.Stream(device=dev)
@@ -429,7 +450,7 @@ def ours_arm(args):
             kt[name] = time_graph(g, kreps, stream) / (kreps * R)
     assert tg.last_device_status(stream) == 0
     t_max = max_over_ranks(t_steps, world)
-    steps_per_s = world * K / t_max
+    steps_per_s = job_throughput(world, K, t_max)
 
     pk, pk_src = peaks()
     hbm = pk["hbm_gbs"]
@@ -464,7 +485,8 @@ def ours_arm(args):
                        "tree_nodes": len(host[0]["parent"]), "tree_depth": sh["depth"],
                        "heads_q_kv": f"{sh['Hq']}/{sh['Hkv']}", "head_dim": sh["D"],
                        "vocab": sh["V"], "topk": sh["k"], "reselect_N": sh["N"],
-                       "l2": f"{R} rotating input sets, ~{R * 40} MB touched per cycle > 126 MB L2",
+                       "l2": f"{R} rotating input sets, ~{R * 40} MB touched per cycle "
+                             + ("> 126 MB L2" if R * 40 > 126 else "(fits in L2)"),
                        "parallelism": f"independent sequences per GPU x{world}"},
             "roofline": roofline, "kernels": kernels, "e2e": e2e,
             "gpu_launches": K * len(KERNELS), "clocks": clocks.summary()}
