@@ -314,7 +314,10 @@ def traffic_record(kernel):
 def sources_hash(names):
     h = hashlib.sha256()
     for name in names:
-        with open(os.path.join(ROOT, "paper_2608_26112_gb300", "csrc", name), "rb") as f:
+        path = os.path.join(ROOT, "paper_2608_26112_gb300", "csrc", name)
+        if not os.path.exists(path):
+            return None
+        with open(path, "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 

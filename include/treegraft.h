@@ -114,7 +114,8 @@ size_t treegraft_tree_attn_workspace_size(int B, int max_nodes, int Hq, int Hkv,
  * k lowest token ids.  Logits must be finite or -inf.
  *
  * logits   [logit_rows, ld] elements of `dtype` (TG_BF16 or TG_F32), row r
- *          at logits + r * ld; V <= ld; V <= 262144 (bf16) or 131072 (fp32).
+ *          at logits + r * ld; V <= ld; V <= 262144 (bf16) or 131072 (fp32);
+ *          aligned to the element size (rows need no further alignment).
  * rows     number of logical rows (rows == 0 is a no-op).
  * row_idx  int32 [rows] of physical rows in [0, logit_rows), or NULL for
  *          rows 0..rows-1 (then rows <= logit_rows).
@@ -183,8 +184,8 @@ size_t treegraft_accept_workspace_size(int B, int n_total);
  *   accept_len = depth(a*) (accepted draft tokens, root excluded);
  *   path = root-first local ids of the root..a* chain, padded with -1 to
  *   path_cap; bonus = am[a*] (the target's next token after a*).
- * target_logits [n_total, ld] of `dtype`; row node_off[b] + v belongs to
- * local node v.  token int32 [n_total] (token[root] ignored).
+ * target_logits [n_total, ld] of `dtype`, aligned to the element size; row
+ * node_off[b] + v belongs to local node v.  token int32 [n_total] (token[root] ignored).
  * path int32 [B, path_cap] (path_cap >= 1); accept_len, bonus int32 [B].
  * ws       scratch of treegraft_accept_workspace_size(B, n_total) bytes,
  *          16-byte aligned, ZERO-FILLED before its first use with this

@@ -27,7 +27,7 @@ struct AcceptSmem {
   float red_v[8];
   uint64_t recv_key[16];  // leader only: per-CTA (max, first position) keys of the row
   int minpos;
-  int tree, off, n, last, bad;
+  int last;
   int par[256];
   int am[256];
   int tok[256];
@@ -52,6 +52,25 @@ __global__ void __launch_bounds__(kScanThreads, 4) accept_kernel(AcceptArgs a, i
 
   uint4 buf[kScanVecs];
   scan_load<T, kAligned>(rowp, c0, c1, buf);
+
+  // The leader resolves the row's tree and fetches the tree's parent and
+  // token arrays while the logits are in flight (any leader may turn out to
+  // be the one that walks the tree).
+  int b = 0, off = 0, n = 0, v_par = -1, v_tok = 0;
+  if (crank == 0) {
+    int lo = 0, hi = a.B - 1;  // last b with node_off[b] <= row
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (__ldg(a.node_off + mid) <= row) lo = mid; else hi = mid - 1;
+    }
+    b = lo;
+    off = __ldg(a.node_off + b);
+    n = __ldg(a.node_off + b + 1) - off;
+    if (n >= 1 && n <= 256 && off >= 0 && off + n <= a.n_total && tid < n) {
+      v_par = __ldg(a.parent + off + tid);
+      v_tok = __ldg(a.token + off + tid);
+    }
+  }
   if (tid == 0) sm.minpos = 0x7FFFFFFF;
   // chunk max, then the lowest position holding it (only threads that hold it search)
   const float tmax = scan_thread_max<T>(buf);
@@ -76,44 +95,29 @@ __global__ void __launch_bounds__(kScanThreads, 4) accept_kernel(AcceptArgs a, i
   if (crank != 0) return;
 
   // leader: publish the argmax, take a ticket for the row's tree
+  const bool bad_tree = (n < 1 || n > 256 || off < 0 || off + n > a.n_total);
   if (tid == 0) {
     uint64_t best = 0;
     for (int c = 0; c < C; ++c) best = sm.recv_key[c] > best ? sm.recv_key[c] : best;
     a.am[row] = (int32_t)key_index(best);
-    // tree of this row: last b with node_off[b] <= row
-    int lo = 0, hi = a.B - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (a.node_off[mid] <= row) lo = mid; else hi = mid - 1;
+    // release: the argmax store above is visible to the CTA that draws the
+    // last ticket; acquire: the last CTA sees every other row's argmax
+    if (bad_tree) {
+      sm.last = 0;  // a malformed extent never touches the ticket
+      raise_status(a.status, kStTree);
+    } else {
+      const int t = atom_add_acq_rel_gpu(&a.tickets[b], 1);
+      sm.last = (t == n - 1);
+      if (sm.last) a.tickets[b] = 0;  // ready for the next call (the next launch orders it)
     }
-    const int b = lo;
-    const int off = a.node_off[b];
-    const int n = a.node_off[b + 1] - off;
-    __threadfence();
-    const int t = atomicAdd(&a.tickets[b], 1);
-    sm.tree = b;
-    sm.off = off;
-    sm.n = n;
-    sm.last = (t == n - 1);
-    if (sm.last) {
-      __threadfence();
-      a.tickets[b] = 0;
-    }
-    sm.bad = (n < 1 || n > 256 || off < 0 || off + n > a.n_total) ? 1 : 0;
-    if (sm.bad) raise_status(a.status, kStTree);
   }
+  sm.par[tid] = v_par;
+  sm.tok[tid] = v_tok;
   __syncthreads();
-  if (!sm.last || sm.bad) return;
+  if (!sm.last) return;
 
   // ---- walk of tree b (this CTA saw every row of the tree finish)
-  const int b = sm.tree, off = sm.off, n = sm.n;
-  int v_par = -1;
-  if (tid < n) {
-    v_par = a.parent[off + tid];
-    sm.par[tid] = v_par;
-    sm.tok[tid] = a.token[off + tid];
-    sm.am[tid] = __ldcg(&a.am[off + tid]);
-  }
+  if (tid < n) sm.am[tid] = __ldcg(&a.am[off + tid]);
   const bool bad = (tid < n) && (tid == 0 ? (v_par != -1) : (v_par < 0 || v_par >= tid));
   if (__syncthreads_or(bad)) {
     if (tid == 0) raise_status(a.status, kStTree);

@@ -66,6 +66,8 @@ extern "C" int treegraft_accept_noalloc(const void* target_logits, int dtype, in
   if (B < 1 || V < 1 || ld < V || n_total < 1 || path_cap < 1 || max_nodes < 1 ||
       max_nodes > TG_MAX_TREE_NODES || (long long)n_total > (long long)B * max_nodes)
     return TG_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(target_logits) & (dtype == TG_BF16 ? 1 : 3)) != 0)
+    return TG_ERR_INVALID_ARG;  // elements must sit at their natural alignment
   // the fixed scratch array bounds the problem size
   if (n_total > kNoAllocMaxNodes || B > kNoAllocMaxTrees) return TG_ERR_UNSUPPORTED;
   if (V > (dtype == TG_BF16 ? 262144 : 131072)) return TG_ERR_UNSUPPORTED;

@@ -173,6 +173,8 @@ int treegraft_expand_topk(const void* logits, int dtype, int logit_rows, int V, 
   if (dtype != TG_BF16 && dtype != TG_F32) return TG_ERR_INVALID_ARG;
   if (rows < 0 || V < 1 || ld < V || logit_rows < 1 || k < 1 || k > V) return TG_ERR_INVALID_ARG;
   if (!row_idx && logit_rows < rows) return TG_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(logits) & (dtype == TG_BF16 ? 1 : 3)) != 0)
+    return TG_ERR_INVALID_ARG;  // elements must sit at their natural alignment
   if (k > TG_MAX_TOPK || V > (dtype == TG_BF16 ? 262144 : 131072)) return TG_ERR_UNSUPPORTED;
   int* st = status_ptr();
   if (!st) return TG_ERR_CUDA;
@@ -247,6 +249,8 @@ int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld, co
     return TG_ERR_INVALID_ARG;
   if (ws_bytes < treegraft_accept_workspace_size(B, n_total) || !aligned16(ws))
     return TG_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(target_logits) & (dtype == TG_BF16 ? 1 : 3)) != 0)
+    return TG_ERR_INVALID_ARG;  // elements must sit at their natural alignment
   if (V > (dtype == TG_BF16 ? 262144 : 131072)) return TG_ERR_UNSUPPORTED;
   int* st = status_ptr();
   if (!st) return TG_ERR_CUDA;

@@ -45,6 +45,15 @@ __device__ __forceinline__ uint64_t make_key(float v, uint32_t idx) {
 __device__ __forceinline__ uint32_t key_index(uint64_t k) { return ~(uint32_t)k; }
 __device__ __forceinline__ float key_value(uint64_t k) { return unord_f32((uint32_t)(k >> 32)); }
 
+// atomicAdd with acquire-release semantics at GPU scope: the caller's earlier
+// writes are visible to whoever later acquires the counter, and writes made
+// before the earlier releases are visible to the caller afterwards.
+__device__ __forceinline__ int atom_add_acq_rel_gpu(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
 __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {

@@ -35,14 +35,18 @@ __global__ void __launch_bounds__(kThreads) rescore_select_kernel(RescoreArgs a)
     return;
   }
   const int v = tid;
-  int p = -1, bad = 0;
-  float e = 0.f;
+  // every per-node input is requested at once; only the strong-row gather
+  // depends on them (parent and token)
+  int p = -1, bad = 0, t = 0;
+  float e = 0.f, w_edge = 0.f;
   bool cand = false;
   if (v < n) {
     p = a.parent[off + v];
+    cand = a.visited[off + v] == 0;
+    t = a.token[off + v];
+    w_edge = a.weak_edge[off + v];
     bad = (v == 0) ? (p != -1) : (p < 0 || p >= v);
     par_s[v] = p;
-    cand = a.visited[off + v] == 0;
   }
   if (__syncthreads_or(bad)) {
     if (tid == 0) raise_status(a.status, kStTree);
@@ -51,14 +55,13 @@ __global__ void __launch_bounds__(kThreads) rescore_select_kernel(RescoreArgs a)
   int bad_tok = 0;
   if (v > 0 && v < n) {
     if (cand) {
-      const int t = a.token[off + v];
       if (t < 0 || t >= a.V) {
         bad_tok = 1;
       } else {
         e = a.strong_lp[(size_t)(off + p) * (size_t)a.ld + t];
       }
     } else {
-      e = a.weak_edge[off + v];
+      e = w_edge;
     }
   }
   if (__syncthreads_or(bad_tok)) {

@@ -86,6 +86,10 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
     return;
   }
   cluster_arrive_relaxed();
+  // the leader's output threads fetch the parent's path score now, while
+  // the logits are in flight
+  float parent_score = 0.f;
+  if (crank == 0 && tid < k) parent_score = __ldg(a.parent_score + row);
   const int per = ((V + C - 1) / C + VW - 1) / VW * VW;
   const int c0 = min(V, crank * per);
   const int c1 = min(V, c0 + per);
@@ -126,17 +130,37 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   const float tv = unord_f32(sm.thr_ord);
   // 3. candidates (only threads whose max reaches the threshold have any)
   if (tmax >= tv) {
-#pragma unroll
-    for (int i = 0; i < kScanVecs; ++i)
-#pragma unroll
-      for (int j = 0; j < VW; ++j) {
-        const float v = vec_elem<T>(buf[i], j);
-        const int pos = scan_pos(c0, i, j, VW);
-        if (pos < c1 && v >= tv) {
-          const int slot = atomicAdd(&sm.ncand, 1);
-          if (slot < kCandMax) sm.cand[slot] = make_key(v, (uint32_t)pos);
-        }
+    auto push = [&](float v, int pos) {
+      if (pos < c1) {
+        const int slot = atomicAdd(&sm.ncand, 1);
+        if (slot < kCandMax) sm.cand[slot] = make_key(v, (uint32_t)pos);
       }
+    };
+    if constexpr (VW == 8) {
+      // one packed compare per element pair; tv is a thread max, so it is
+      // exactly representable in bf16
+      const __nv_bfloat162 tv2 = __float2bfloat162_rn(tv);
+#pragma unroll
+      for (int i = 0; i < kScanVecs; ++i)
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const uint32_t x = vec_word(buf[i], w);
+          const uint32_t mk = __hge2_mask(*reinterpret_cast<const __nv_bfloat162*>(&x), tv2);
+          if (mk) {
+            const int pos = scan_pos(c0, i, 2 * w, VW);
+            if (mk & 0xFFFFu) push(bf16_lo(x), pos);
+            if (mk >> 16) push(bf16_hi(x), pos + 1);
+          }
+        }
+    } else {
+#pragma unroll
+      for (int i = 0; i < kScanVecs; ++i)
+#pragma unroll
+        for (int j = 0; j < VW; ++j) {
+          const float v = vec_elem<T>(buf[i], j);
+          if (v >= tv) push(v, scan_pos(c0, i, j, VW));
+        }
+    }
   }
   __syncthreads();
   int nc = sm.ncand;
@@ -199,12 +223,21 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   if (crank != 0) return;
 
   // ---- leader: merge the C partials
-  if (tid == 0) {
-    float M = sm.recv_m[0], S = sm.recv_s[0];
-    for (int c = 1; c < C; ++c) lse_merge(M, S, sm.recv_m[c], sm.recv_s[c]);
-    const float lse = (M == __int_as_float(0xff800000)) ? M : M + log2f(S) * kLn2;
-    sm.lse = lse;
-    if (a.lse_out) a.lse_out[row] = lse;
+  if (warp == 0) {
+    // lse over the C partials: one (max, sum) per lane, shuffle tree
+    float M = lane < C ? sm.recv_m[lane] : __int_as_float(0xff800000);
+    float S = lane < C ? sm.recv_s[lane] : 0.f;
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, M, o);
+      const float s2 = __shfl_xor_sync(0xffffffffu, S, o);
+      lse_merge(M, S, m2, s2);
+    }
+    if (lane == 0) {
+      const float lse = (M == __int_as_float(0xff800000)) ? M : M + log2f(S) * kLn2;
+      sm.lse = lse;
+      if (a.lse_out) a.lse_out[row] = lse;
+    }
   }
   for (int t = tid; t < C * k; t += kScanThreads) {
     const uint64_t mine = sm.recv_top[t];
@@ -221,7 +254,7 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
     const size_t o = (size_t)row * k + tid;
     a.tok[o] = (int32_t)key_index(key);
     a.logprob[o] = lp;
-    a.score[o] = __fadd_rn(a.parent_score[row], lp);
+    a.score[o] = __fadd_rn(parent_score, lp);
   }
 }
 
