@@ -49,8 +49,11 @@ constexpr int kRegion = 128 * 128;  // 128 rows x 128 bytes: one swizzled operan
 constexpr int kMaxSplits = 8;
 constexpr float kLn2 = 0.6931471805599453f;
 
-enum { BAR_KV_FULL = 0, BAR_KV_EMPTY = 2, BAR_Q_FULL = 4, BAR_S_FULL = 5 /* 2 buffers */,
-       BAR_P_FULL = 7, BAR_O_DONE = 8, kNumBars = 9 };
+// K and V have their own rings: a K stage is free once its S = Q K^T
+// product is done, a V stage once its PV product is, so the next K tile is
+// requested well before the current PV finishes.
+enum { BAR_K_FULL = 0, BAR_V_FULL = 2, BAR_K_EMPTY = 4, BAR_V_EMPTY = 6, BAR_Q_FULL = 8,
+       BAR_S_FULL = 9 /* 2 buffers */, BAR_P_FULL = 11, BAR_O_DONE = 12, kNumBars = 13 };
 
 constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
@@ -72,17 +75,19 @@ struct Layout {
   static constexpr int kOffMisc = align_up(kOffBar + kNumBars * 8, 16);    // tmem addr, flag
   static constexpr int kBytes = kOffMisc + 16;
   static constexpr int kAlloc = kBytes + 1024;                       // 1024-byte alignment slack
-  // Partial rows of the combine, written once every MMA of the CTA is done,
-  // over the Q / K tiles: a row is [O (D fp32) | m (base 2) | l | 2 pad].
-  static constexpr int kRowFloats = D + 4;
-  static constexpr int kSlabBytes = kBM * kRowFloats * 4;            // one CTA's partial rows
-  static constexpr int kOffStage = 0;
-  static_assert(kOffStage + kSlabBytes <= kTileEnd, "staging fits the tiles");
+  // One CTA's partial rows in the workspace, laid out so that a warp (32
+  // consecutive rows) writes and reads 512 contiguous bytes: O as
+  // [D / 4][kBM] float4 (column group major), then m[kBM] (base 2) and
+  // l[kBM], then kBM * 2 spare floats.
+  static constexpr int kSlabFloats = kBM * (D + 4);
+  static constexpr int kSlabBytes = kSlabFloats * 4;
+  static constexpr int kSlabM = kBM * D;        // float offset of m[]
+  static constexpr int kSlabL = kBM * (D + 1);  // float offset of l[]
   static_assert(kAlloc <= 227 * 1024, "shared memory budget");
   static_assert(kOffQ % 1024 == 0 && kOffK % 1024 == 0 && kOffV % 1024 == 0 && kOffP % 1024 == 0,
                 "128-byte-swizzled operand tiles need 1024-byte alignment");
   static_assert(kOffBar % 8 == 0 && kOffMisc % 16 == 0, "mbarrier / scalar alignment");
-  static_assert((kRowFloats * 4) % 16 == 0 && kSlabBytes % 16 == 0, "float4 staging rows");
+  static_assert(kSlabBytes % 16 == 0, "float4 slab");
 };
 
 // 32 mask bits of one node for tree slots [b0, b0 + 32): slot < 0 is the
@@ -138,7 +143,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + L::kOffAnc);
   float* red_max = reinterpret_cast<float*>(smem + L::kOffRedMax);
   float* red_l = reinterpret_cast<float*>(smem + L::kOffRedL);
-  float* stage_rows = reinterpret_cast<float*>(smem + L::kOffStage);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kOffMisc);
   int* bad_flag = reinterpret_cast<int*>(smem + L::kOffMisc + 4);
   const uint32_t bar0 = smem_u32(smem + L::kOffBar);
@@ -156,15 +160,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---- barriers; the first K/V copies go out before any global read returns
   const int kv_row0 = (b * a.Hkv + h) * a.S_max;
-  auto load_kv = [&](int it) {  // it-th tile of this split = tile split + it * S_kv
+  auto load_k = [&](int it) {  // it-th tile of this split = tile split + it * S_kv
     const int st = it & 1;
-    mbar_arrive_expect_tx(bar(BAR_KV_FULL + st), 2 * L::kKVBytes);
+    mbar_arrive_expect_tx(bar(BAR_K_FULL + st), L::kKVBytes);
     const int y = kv_row0 + (split + it * S_kv) * kBN;
 #pragma unroll
-    for (int c = 0; c < D / 64; ++c) {
-      tma_load_2d(k_base + st * L::kKVBytes + c * kRegion, &tm_k, c * 64, y, bar(BAR_KV_FULL + st));
-      tma_load_2d(v_base + st * L::kKVBytes + c * kRegion, &tm_v, c * 64, y, bar(BAR_KV_FULL + st));
-    }
+    for (int c = 0; c < D / 64; ++c)
+      tma_load_2d(k_base + st * L::kKVBytes + c * kRegion, &tm_k, c * 64, y, bar(BAR_K_FULL + st));
+  };
+  auto load_v = [&](int it) {
+    const int st = it & 1;
+    mbar_arrive_expect_tx(bar(BAR_V_FULL + st), L::kKVBytes);
+    const int y = kv_row0 + (split + it * S_kv) * kBN;
+#pragma unroll
+    for (int c = 0; c < D / 64; ++c)
+      tma_load_2d(v_base + st * L::kKVBytes + c * kRegion, &tm_v, c * 64, y, bar(BAR_V_FULL + st));
   };
   // Early copies are issued only for boxes that start inside the tensors (a
   // box past the last row is never requested), and every issued copy is
@@ -183,8 +193,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool q_early = (b == 0) && (r0 / G < a.n_total);
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(bar(BAR_KV_FULL + s), 1);
-      mbar_init(bar(BAR_KV_EMPTY + s), 1);
+      mbar_init(bar(BAR_K_FULL + s), 1);
+      mbar_init(bar(BAR_V_FULL + s), 1);
+      mbar_init(bar(BAR_K_EMPTY + s), 1);
+      mbar_init(bar(BAR_V_EMPTY + s), 1);
       mbar_init(bar(BAR_S_FULL + s), 1);
     }
     mbar_init(bar(BAR_Q_FULL), 1);
@@ -198,7 +210,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (q_early) load_q(r0 / G);
 #pragma unroll
     for (int s = 0; s < kStages; ++s)
-      if (kv_early[s]) load_kv(s);  // used when this split has that many tiles
+      if (kv_early[s]) {  // used when this split has that many tiles
+        load_k(s);
+        load_v(s);
+      }
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), 512);  // S buffers: [0,128) [128,256); O: [256, 256 + D)
@@ -223,7 +238,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (tid == 0) {
       bool ok = true;
       for (int s = 0; s < kStages; ++s)
-        if (kv_early[s]) ok = mbar_wait(bar(BAR_KV_FULL + s), 0) && ok;
+        if (kv_early[s]) {
+          ok = mbar_wait(bar(BAR_K_FULL + s), 0) && ok;
+          ok = mbar_wait(bar(BAR_V_FULL + s), 0) && ok;
+        }
       if (q_early) ok = mbar_wait(bar(BAR_Q_FULL), 0) && ok;
       if (!ok) raise_status(a.status, kStTimeout);
       if (bad_shape && split == 0 && blockIdx.y == 0) raise_status(a.status, kStTree);
@@ -235,16 +253,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------ TMA producer
-    if (lane == 0) {
+    if (lane < 2) {
       // real tiles always lie inside the tensors, so an early stage was issued
-      // for each of the first min(nt, kStages) tiles
+      // for each of the first min(nt, kStages) tiles.  Lane 0 refills K
+      // (after the S product of the tile two back), lane 1 refills V (after
+      // its PV product).
+      const int empty = lane == 0 ? BAR_K_EMPTY : BAR_V_EMPTY;
       for (int it = kStages; it < nt; ++it) {
         const int st = it & 1;
-        if (!mbar_wait(bar(BAR_KV_EMPTY + st), ((it >> 1) - 1) & 1)) {
+        if (!mbar_wait(bar(empty + st), ((it >> 1) - 1) & 1)) {
           raise_status(a.status, kStTimeout);
           break;
         }
-        load_kv(it);
+        if (lane == 0) load_k(it); else load_v(it);
       }
     }
     __syncwarp();
@@ -260,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // S buffer it&1 was last read by the softmax of tile it-2, whose
           // P_FULL phase was awaited before PV(it-2) was issued
           const int st = it & 1;
-          ok = mbar_wait(bar(BAR_KV_FULL + st), (it >> 1) & 1);
+          ok = mbar_wait(bar(BAR_K_FULL + st), (it >> 1) & 1);
           if (!ok) break;
           tc_fence_after();
 #pragma unroll
@@ -271,10 +292,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                        smem_desc_sw128(ka, 16, 1024), kIdS, kk > 0 ? 1u : 0u);
           }
           tc_commit(bar(BAR_S_FULL + st));
+          tc_commit(bar(BAR_K_EMPTY + st));
         }
         if (it > 0) {
           const int jt = it - 1, sp = jt & 1;
-          ok = mbar_wait(bar(BAR_P_FULL), jt & 1);
+          ok = mbar_wait(bar(BAR_P_FULL), jt & 1) && mbar_wait(bar(BAR_V_FULL + sp), (jt >> 1) & 1);
           if (!ok) break;
           tc_fence_after();
 #pragma unroll
@@ -285,7 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                        kIdO, (jt > 0 || kk > 0) ? 1u : 0u);
           }
           tc_commit(bar(BAR_O_DONE));
-          tc_commit(bar(BAR_KV_EMPTY + sp));
+          tc_commit(bar(BAR_V_EMPTY + sp));
         }
       }
       if (!ok) raise_status(a.status, kStTimeout);
@@ -398,7 +420,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (tile_key0 + kBN > Lk) {
         // last tile of the sequence: V rows past the end may hold anything;
         // zero them so that 0-weight rows contribute exactly 0
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_KV_FULL + st), (it >> 1) & 1));
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_V_FULL + st), (it >> 1) & 1));
         if (!ok) continue;
         if (tile_key0 + r >= Lk && half < D / 64) {
 #pragma unroll
@@ -428,7 +450,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // speculative K/V copies this split did not use land in the buffers the
     // staging below reuses: wait for them first
     for (int it = nt; it < kStages; ++it)
-      if (kv_early[it] && !mbar_wait(bar(BAR_KV_FULL + it), 0)) ok = false;
+      if (kv_early[it] && !(mbar_wait(bar(BAR_K_FULL + it), 0) && mbar_wait(bar(BAR_V_FULL + it), 0)))
+        ok = false;
     if (nt == 0 && q_early && !mbar_wait(bar(BAR_Q_FULL), 0)) ok = false;  // no MMA waited it
     ok = __all_sync(0xffffffffu, ok);
     if (!ok && lane == 0) raise_status(a.status, kStTimeout);
@@ -463,8 +486,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (half == 0 && uu < n && a.lse_out)
         a.lse_out[orow] = live ? (m_run * sl2 + log2f(l_tot)) * kLn2 : NEG_INF;
     } else {
-      // ---- stage this row's partial: [O (D fp32) | m (base 2) | l | pad]
-      float* row = stage_rows + r * L::kRowFloats;
+      // ---- this row's partial straight into the workspace:
+      //      [O (D fp32) | m (base 2) | l | pad], read back after the cluster barrier
+      const size_t unit = (size_t)blockIdx.z * gridDim.y + blockIdx.y;
+      float* slab = reinterpret_cast<float*>(a.ws) + (unit * (size_t)S_kv + (size_t)split) * L::kSlabFloats;
+      float4* slab4 = reinterpret_cast<float4*>(slab);
       // tcgen05.ld / wait::ld are warp-collective: the condition must be the
       // same for the 32 lanes (ok and nt are); per-row liveness only selects
       // what is stored
@@ -475,18 +501,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld32f(tmem_O + lane_off + half * DH + c * 32, o);
           tc_wait_ld();
 #pragma unroll
-          for (int q = 0; q < 32; q += 4)
-            *reinterpret_cast<float4*>(row + half * DH + c * 32 + q) =
-                live ? make_float4(o[q], o[q + 1], o[q + 2], o[q + 3])
-                     : make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int q = 0; q < 8; ++q)
+            __stcg(slab4 + ((half * DH + c * 32) / 4 + q) * kBM + r,
+                   live ? make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3])
+                        : make_float4(0.f, 0.f, 0.f, 0.f));
         }
       } else {
-        for (int c = 0; c < DH; c += 4)
-          *reinterpret_cast<float4*>(row + half * DH + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int c4 = 0; c4 < DH / 4; ++c4)
+          __stcg(slab4 + (half * DH / 4 + c4) * kBM + r, make_float4(0.f, 0.f, 0.f, 0.f));
       }
       if (half == 0) {
-        row[D] = live ? m_run * sl2 : NEG_INF;
-        row[D + 1] = live ? l_tot : 0.f;
+        __stcg(slab + L::kSlabM + r, live ? m_run * sl2 : NEG_INF);
+        __stcg(slab + L::kSlabL + r, live ? l_tot : 0.f);
       }
     }
   }
@@ -500,27 +526,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
 
-  // ---- combine through L2: publish this CTA's partial rows, then reduce the owned rows
-  __syncthreads();  // TMEM reads are done; the staged rows are complete
+  // ---- combine through L2: every CTA has written its partial rows; the
+  // cluster barrier (release / acquire at cluster scope) makes them visible
+  // to the other CTAs of the cluster, and ends this CTA's TMEM reads
+  cluster.sync();
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
   const size_t unit = (size_t)blockIdx.z * gridDim.y + blockIdx.y;
-  float* slabs = reinterpret_cast<float*>(a.ws) + unit * (size_t)S_kv * (L::kSlabBytes / 4);
-  {
-    float4* dst = reinterpret_cast<float4*>(slabs + (size_t)split * (L::kSlabBytes / 4));
-    const float4* src = reinterpret_cast<const float4*>(stage_rows);
-    for (int i = tid; i < L::kSlabBytes / 16; i += kThreads) __stcg(dst + i, src[i]);
-  }
-  __threadfence();
-  cluster.sync();  // every CTA of the cluster has published its rows
+  const float* slabs = reinterpret_cast<const float*>(a.ws) + unit * (size_t)S_kv * L::kSlabFloats;
   const int rpc = (kBM + S_kv - 1) / S_kv;  // tile rows owned by each CTA of the cluster
   const int row_lo = split * rpc;
   const int my_rows = max(0, min(kBM, row_lo + rpc) - row_lo);
   constexpr int CG = D / 8;  // 8-column groups per row
+  // items run row-fastest so that a warp reads consecutive rows of one
+  // column group: contiguous in the slab layout
   for (int item = tid; item < my_rows * CG; item += kThreads) {
-    const int rr = row_lo + item / CG, c8 = item % CG;
+    const int rr = row_lo + item % my_rows, c8 = item / my_rows;
     const int rg = r0 + rr;
     const int uu = rg / G, g = rg % G;
     if (uu >= n) continue;
@@ -530,11 +553,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int sp = 0; sp < kMaxSplits; ++sp) {
       if (sp < S_kv) {
-        const float* src = slabs + (size_t)sp * (L::kSlabBytes / 4) + rr * L::kRowFloats;
-        mv[sp] = __ldcg(src + D);
-        lv[sp] = __ldcg(src + D + 1);
-        ov[sp][0] = __ldcg(reinterpret_cast<const float4*>(src + c8 * 8));
-        ov[sp][1] = __ldcg(reinterpret_cast<const float4*>(src + c8 * 8 + 4));
+        const float* src = slabs + (size_t)sp * L::kSlabFloats;
+        const float4* src4 = reinterpret_cast<const float4*>(src);
+        mv[sp] = __ldcg(src + L::kSlabM + rr);
+        lv[sp] = __ldcg(src + L::kSlabL + rr);
+        ov[sp][0] = __ldcg(src4 + (2 * c8) * kBM + rr);
+        ov[sp][1] = __ldcg(src4 + (2 * c8 + 1) * kBM + rr);
       }
     }
     float M = NEG_INF;
