@@ -121,6 +121,79 @@ __device__ __forceinline__ void softmax_bar() {
   asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
 }
 
+// Columns one combine item covers with S splits: wide enough that a single
+// pass of the CTA's threads covers the rows it owns (ceil(128 / S) rows of
+// D columns), narrow enough that the S x COLS loaded floats stay in
+// registers, so every load of an item is in flight at once.
+template <int S>
+constexpr int combine_cols() {
+  return S <= 3 ? 32 : (S <= 6 ? 16 : 8);
+}
+
+// Merge the S partial rows of the rows this CTA owns (Sec. 3.1 attention as
+// a softmax over the union of the splits' keys): o = sum_s w_s O_s / sum_s
+// w_s l_s with w_s = 2^(m_s - max_s m_s), lse = ln 2 (max + log2 sum).
+template <int D, int S>
+__device__ __forceinline__ void combine_rows(const float* slabs, int split, int r0, int G, int n,
+                                             int off, int h, const AttnArgs& a) {
+  using L = Layout<D>;
+  constexpr int COLS = combine_cols<S>() < D ? combine_cols<S>() : D;
+  constexpr int NV = COLS / 4;  // float4 per split per item
+  constexpr int CG = D / COLS;
+  const float NEG_INF = __int_as_float(0xff800000);
+  const int rpc = (kBM + S - 1) / S;  // tile rows owned by each CTA of the cluster
+  const int row_lo = split * rpc;
+  const int my_rows = max(0, min(kBM, row_lo + rpc) - row_lo);
+  // items run row-fastest so that a warp reads consecutive rows of one
+  // column group: contiguous in the slab layout
+  for (int item = threadIdx.x; item < my_rows * CG; item += kThreads) {
+    const int rr = row_lo + item % my_rows, cg = item / my_rows;
+    const int rg = r0 + rr;
+    const int uu = rg / G, g = rg % G;
+    if (uu >= n) continue;
+    float mv[S], lv[S];
+    float4 ov[S][NV];
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) {
+      const float* src = slabs + (size_t)sp * L::kSlabFloats;
+      const float4* src4 = reinterpret_cast<const float4*>(src);
+      mv[sp] = __ldcg(src + L::kSlabM + rr);
+      lv[sp] = __ldcg(src + L::kSlabL + rr);
+#pragma unroll
+      for (int q = 0; q < NV; ++q) ov[sp][q] = __ldcg(src4 + (cg * NV + q) * kBM + rr);
+    }
+    float M = NEG_INF;
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) M = fmaxf(M, mv[sp]);
+    float Ls = 0.f;
+    float acc[COLS];
+#pragma unroll
+    for (int q = 0; q < COLS; ++q) acc[q] = 0.f;
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) {
+      const float w = (mv[sp] == NEG_INF) ? 0.f : ex2(mv[sp] - M);
+      Ls += w * lv[sp];
+#pragma unroll
+      for (int q = 0; q < NV; ++q) {
+        acc[4 * q + 0] += w * ov[sp][q].x;
+        acc[4 * q + 1] += w * ov[sp][q].y;
+        acc[4 * q + 2] += w * ov[sp][q].z;
+        acc[4 * q + 3] += w * ov[sp][q].w;
+      }
+    }
+    const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
+    const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
+    uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + cg * COLS);
+#pragma unroll
+    for (int q = 0; q < COLS / 8; ++q)
+      dst[q] = make_uint4(pack_bf16(acc[8 * q + 0] * inv, acc[8 * q + 1] * inv),
+                          pack_bf16(acc[8 * q + 2] * inv, acc[8 * q + 3] * inv),
+                          pack_bf16(acc[8 * q + 4] * inv, acc[8 * q + 5] * inv),
+                          pack_bf16(acc[8 * q + 6] * inv, acc[8 * q + 7] * inv));
+    if (cg == 0 && a.lse_out) a.lse_out[orow] = (M == NEG_INF) ? M : (M + log2f(Ls)) * kLn2;
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
@@ -536,63 +609,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   const size_t unit = (size_t)blockIdx.z * gridDim.y + blockIdx.y;
   const float* slabs = reinterpret_cast<const float*>(a.ws) + unit * (size_t)S_kv * L::kSlabFloats;
-  const int rpc = (kBM + S_kv - 1) / S_kv;  // tile rows owned by each CTA of the cluster
-  const int row_lo = split * rpc;
-  const int my_rows = max(0, min(kBM, row_lo + rpc) - row_lo);
-  constexpr int CG = D / 8;  // 8-column groups per row
-  // items run row-fastest so that a warp reads consecutive rows of one
-  // column group: contiguous in the slab layout
-  for (int item = tid; item < my_rows * CG; item += kThreads) {
-    const int rr = row_lo + item % my_rows, c8 = item / my_rows;
-    const int rg = r0 + rr;
-    const int uu = rg / G, g = rg % G;
-    if (uu >= n) continue;
-    // issue every load before using any of them
-    float mv[kMaxSplits], lv[kMaxSplits];
-    float4 ov[kMaxSplits][2];
-#pragma unroll
-    for (int sp = 0; sp < kMaxSplits; ++sp) {
-      if (sp < S_kv) {
-        const float* src = slabs + (size_t)sp * L::kSlabFloats;
-        const float4* src4 = reinterpret_cast<const float4*>(src);
-        mv[sp] = __ldcg(src + L::kSlabM + rr);
-        lv[sp] = __ldcg(src + L::kSlabL + rr);
-        ov[sp][0] = __ldcg(src4 + (2 * c8) * kBM + rr);
-        ov[sp][1] = __ldcg(src4 + (2 * c8 + 1) * kBM + rr);
-      }
-    }
-    float M = NEG_INF;
-#pragma unroll
-    for (int sp = 0; sp < kMaxSplits; ++sp)
-      if (sp < S_kv) M = fmaxf(M, mv[sp]);
-    float Ls = 0.f;
-    float acc[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-#pragma unroll
-    for (int sp = 0; sp < kMaxSplits; ++sp) {
-      if (sp < S_kv) {
-        const float w = (mv[sp] == NEG_INF) ? 0.f : ex2(mv[sp] - M);
-        Ls += w * lv[sp];
-        acc[0] += w * ov[sp][0].x;
-        acc[1] += w * ov[sp][0].y;
-        acc[2] += w * ov[sp][0].z;
-        acc[3] += w * ov[sp][0].w;
-        acc[4] += w * ov[sp][1].x;
-        acc[5] += w * ov[sp][1].y;
-        acc[6] += w * ov[sp][1].z;
-        acc[7] += w * ov[sp][1].w;
-      }
-    }
-    const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
-    const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
-    uint4 pk;
-    pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-    pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-    pk.z = pack_bf16(acc[4] * inv, acc[5] * inv);
-    pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
-    *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c8 * 8) = pk;
-    if (c8 == 0 && a.lse_out) a.lse_out[orow] = (M == NEG_INF) ? M : (M + log2f(Ls)) * kLn2;
+  switch (S_kv) {
+    case 2: combine_rows<D, 2>(slabs, split, r0, G, n, off, h, a); break;
+    case 3: combine_rows<D, 3>(slabs, split, r0, G, n, off, h, a); break;
+    case 4: combine_rows<D, 4>(slabs, split, r0, G, n, off, h, a); break;
+    case 5: combine_rows<D, 5>(slabs, split, r0, G, n, off, h, a); break;
+    case 6: combine_rows<D, 6>(slabs, split, r0, G, n, off, h, a); break;
+    case 7: combine_rows<D, 7>(slabs, split, r0, G, n, off, h, a); break;
+    default: combine_rows<D, 8>(slabs, split, r0, G, n, off, h, a); break;
   }
 }
 
