@@ -203,7 +203,7 @@ def make_trees(rng, shape: dict):
 
 def make_workload(name_or_shape, seed: int = 0, *, kv_tail: str = "zero",
                   with_logits: bool = True, with_strong: bool = True,
-                  S_max: int | None = None) -> dict:
+                  S_max: int | None = None, kv_trees: list[int] | None = None) -> dict:
     """All inputs of one verify-and-grow step for a named workload (or a
     shape dict), drawn from PCG64(seed).
 
@@ -218,6 +218,9 @@ def make_workload(name_or_shape, seed: int = 0, *, kv_tail: str = "zero",
         stored edge log-probs and a stronger drafter's log-probs, drawn
         log-prob shaped (mean -ln V - 4.5, sd 3, capped at 0),
       visited (uint8 [n_total]): nodes of depth <= 2 marked visited.
+    With kv_trees, K/V are drawn only for those trees and k_cache / v_cache
+    hold just their rows ([len(kv_trees), Hkv, S_max, D]); every other tree's
+    K/V is all zeros (large serving batches stay cheap to build).
     """
     shape = dict(WORKLOADS[name_or_shape]) if isinstance(name_or_shape, str) else dict(name_or_shape)
     rng = make_rng(seed)
@@ -233,8 +236,14 @@ def make_workload(name_or_shape, seed: int = 0, *, kv_tail: str = "zero",
     out = dict(shape=shape, parent=parent, token=token, node_off=node_off,
                prefix_len=np.asarray(Ps, dtype=np.int32), S_max=S_max)
     out["q"] = f32_to_bf16_bits(normal_f32(rng, (n_total, Hq, D)))
-    out["k_cache"] = kv_cache(rng, B, Hkv, S_max, D, valid, kv_tail)
-    out["v_cache"] = kv_cache(rng, B, Hkv, S_max, D, valid, kv_tail)
+    if kv_trees is None:
+        out["k_cache"] = kv_cache(rng, B, Hkv, S_max, D, valid, kv_tail)
+        out["v_cache"] = kv_cache(rng, B, Hkv, S_max, D, valid, kv_tail)
+    else:
+        sel = [valid[b] for b in kv_trees]
+        out["kv_trees"] = list(kv_trees)
+        out["k_cache"] = kv_cache(rng, len(sel), Hkv, S_max, D, sel, kv_tail)
+        out["v_cache"] = kv_cache(rng, len(sel), Hkv, S_max, D, sel, kv_tail)
     # depth <= 2 nodes are marked visited (older nodes of a shared tree)
     vis = np.zeros(n_total, dtype=np.uint8)
     for b in range(B):

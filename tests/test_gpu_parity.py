@@ -374,3 +374,89 @@ def test_graft_step_pipeline(dev):
     rp, rA, rb = O.accept(tl_bits, token, parent, g["node_off"], n2, bf16=True)
     np.testing.assert_array_equal(path, rp)
     assert A[0] == rA[0] and bonus[0] == rb[0]
+
+
+# ------------------------------------------------------------------ serving sweep
+
+def _serving_kv(wl, dev):
+    """Device K/V caches of a serving workload built with kv_trees: the
+    drawn trees' rows scattered into zero caches."""
+    sh = wl["shape"]
+    B, Hkv, D = sh["B"], sh["Hkv"], sh["D"]
+    k = torch.zeros((B, Hkv, wl["S_max"], D), dtype=torch.bfloat16, device=dev)
+    v = torch.zeros_like(k)
+    for i, b in enumerate(wl["kv_trees"]):
+        k[b] = _dev.bf16(wl["k_cache"][i], dev)
+        v[b] = _dev.bf16(wl["v_cache"][i], dev)
+    return k, v
+
+
+@pytest.mark.parametrize("B", [4, 16, 64])
+def test_tree_attn_serving_sweep(dev, B):
+    """Ragged serving batch: prefixes log-uniform in 512-32768, trees of
+    32-256 nodes, depth 4-10, GQA 32/8.  Three trees carry random K/V and
+    are checked against the oracle; every other tree has all-zero K/V, so
+    its outputs are exactly 0 and its lse is ln(P + depth(u) + 1) - the
+    number of keys the Algorithm 3 mask lets node u see."""
+    sh = synth.serving_shape(B, seed=0)
+    drawn = sorted({0, B // 2, B - 1})
+    wl = synth.make_workload(sh, seed=B, with_logits=False, with_strong=False, kv_trees=drawn)
+    k, v = _serving_kv(wl, dev)
+    q = _dev.bf16(wl["q"], dev)
+    lse = torch.full((q.shape[0], q.shape[1]), float("nan"), device=dev)
+    out, _ = tg.tree_attn(q, k, v, _dev.i32(wl["prefix_len"], dev), _dev.i32(wl["parent"], dev),
+                          _dev.i32(wl["node_off"], dev), _dev.max_nodes(wl), lse_out=lse)
+    _status_clean()
+    o = _dev.bf16_to_np(out)
+    lse = lse.cpu().numpy().astype(np.float64)
+    off = wl["node_off"]
+    for i, b in enumerate(drawn):
+        a, e = int(off[b]), int(off[b + 1])
+        ref_o, ref_lse = O.tree_attention(wl["q"][a:e], wl["k_cache"][i:i + 1],
+                                          wl["v_cache"][i:i + 1], wl["prefix_len"][b:b + 1],
+                                          wl["parent"][a:e], [0, e - a], Hkv=sh["Hkv"])
+        _check_attn(wl, o[a:e], lse[a:e], ref_o, ref_lse)
+    for b in range(B):
+        if b in drawn:
+            continue
+        a, e = int(off[b]), int(off[b + 1])
+        assert np.all(o[a:e] == 0.0)
+        count = int(wl["prefix_len"][b]) + O.node_depth(wl["parent"][a:e]) + 1
+        np.testing.assert_allclose(lse[a:e], np.log(count)[:, None] * np.ones((1, sh["Hq"])),
+                                   atol=LSE_ABS, rtol=0)
+
+
+def test_accept_serving_sweep(dev):
+    """accept on an 8-tree ragged serving batch (n 32-256, depth 4-10) with
+    bf16 target logits over 128256 tokens, bumps planted at +40 so that long
+    paths occur; bit-exact against the oracle."""
+    sh = synth.serving_shape(8, seed=1)
+    wl = synth.make_workload(sh, seed=8, with_strong=False, with_logits=False, kv_trees=[])
+    rng = synth.make_rng(88)
+    lg = synth.normal_f32(rng, (len(wl["parent"]), sh["V"]), 3.0)
+    off = wl["node_off"]
+    for b in range(sh["B"]):
+        a, e = int(off[b]), int(off[b + 1])
+        synth.plant_child_bump(rng, lg, wl["parent"][a:e], wl["token"][a:e], np.arange(a, e),
+                               prob=0.9, bump=40.0)
+    wl["logits"] = synth.f32_to_bf16_bits(lg)
+    cap = 16
+    got = _run_accept(wl, dev, cap)
+    ref = O.accept(wl["logits"], wl["token"], wl["parent"], wl["node_off"], cap, bf16=True)
+    for g, r in zip(got[:3], ref):
+        np.testing.assert_array_equal(g, r)
+    assert ref[1].max() >= 2
+
+
+def test_expand_topk_serving_rows(dev):
+    """expand_topk over 128 frontier rows picked by row_idx from 512 bf16
+    logit rows over 128256 tokens (k = 10), as a serving step expands the
+    frontier of every tree in the batch."""
+    sh = synth.serving_shape(8, seed=2)
+    rng = synth.make_rng(9)
+    lg = synth.f32_to_bf16_bits(synth.normal_f32(rng, (512, sh["V"]), 3.0))
+    rows = np.sort(synth.make_rng(77).choice(512, size=128, replace=False)).astype(np.int32)
+    ps = -np.abs(synth.normal_f32(rng, (128,), 4.0))
+    got = _run_expand(_dev.bf16(lg, dev), ps, sh["k"], dev, row_idx=rows)
+    ref = O.expand_topk(lg, ps, sh["k"], row_idx=rows, bf16=True)
+    _check_expand(got, ref)
