@@ -133,7 +133,7 @@ def alloc_outputs(d, sh, dev):
         alen=torch.empty(1, dtype=torch.int32, device=dev),
         bonus=torch.empty(1, dtype=torch.int32, device=dev),
         ws=tg.accept_workspace(1, n, dev),
-        attn_ws=torch.empty(max(16, tg.tree_attn_workspace_size(
+        attn_ws=torch.zeros(max(16, tg.tree_attn_workspace_size(
             1, n, d["q"].shape[1], d["k"].shape[1], d["q"].shape[2])), dtype=torch.uint8,
             device=dev))
 

@@ -77,9 +77,12 @@ typedef enum { TG_BF16 = 0, TG_F32 = 1 } tg_dtype;
  * scale    softmax scale; 0 selects D^-1/2.
  * out      bf16 [n_total, Hq, D];  lse_out fp32 [n_total, Hq] or NULL.
  * ws       scratch of treegraft_tree_attn_workspace_size(B, max_nodes, Hq,
- *          Hkv, D) bytes, 16-byte aligned: partial rows of the split-KV
- *          combine (needs no initialisation).  Calls sharing one ws must not
- *          overlap on the GPU.
+ *          Hkv, D) bytes, 16-byte aligned, ZERO-FILLED before its first use:
+ *          split counters (returned to zero by every call) and the partial
+ *          rows of the split-KV combine.  Calls sharing one ws must not
+ *          overlap on the GPU.  When the whole grid fits on the GPU at once
+ *          the launch is cooperative and the splits of a work item meet on
+ *          those counters (a bounded wait: TG_ERR_TIMEOUT, never a hang).
  * Errors: TG_ERR_INVALID_ARG (null pointer, bad sizes, misaligned q/k/v),
  *   TG_ERR_UNSUPPORTED (D or G outside the list), TG_ERR_CUDA.  A malformed
  *   tree sets TG_ERR_DEVICE_TREE; its rows of `out` and `lse_out` are then

@@ -134,7 +134,7 @@ def tree_attn(q, k_cache, v_cache, prefix_len, parent, node_off, max_nodes, *, s
     if lse_out is not None:
         _need(lse_out, torch.float32, "lse_out")
     if ws is None:
-        ws = torch.empty(max(16, tree_attn_workspace_size(B, max_nodes, Hq, Hkv, D)),
+        ws = torch.zeros(max(16, tree_attn_workspace_size(B, max_nodes, Hq, Hkv, D)),
                          dtype=torch.uint8, device=q.device)
     _need(ws, torch.uint8, "ws")
     st = lib().treegraft_tree_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(prefix_len),

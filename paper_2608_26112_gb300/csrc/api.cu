@@ -99,7 +99,7 @@ extern "C" {
 size_t treegraft_tree_attn_workspace_size(int B, int max_nodes, int Hq, int Hkv, int D) {
   if (B < 1 || max_nodes < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || (D != 64 && D != 128)) return 0;
   const int mtiles = ((Hq / Hkv) * max_nodes + 127) / 128;
-  return tree_attn_ws_bytes(D, B, Hkv, mtiles, 8);
+  return tree_attn_ws_bytes(D, B, Hkv, mtiles, kAttnMaxSplits);
 }
 
 int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
@@ -155,11 +155,12 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
   a.lse_out = lse_out;
   a.status = st;
   const int mtiles = (G * max_nodes + 127) / 128;
-  const int splits = tree_attn_pick_splits(D, B, Hkv, mtiles, S_max, device_sm_count());
-  const size_t need = tree_attn_ws_bytes(D, B, Hkv, mtiles, splits);
+  const AttnPlan plan = tree_attn_plan(D, B, Hkv, mtiles, S_max, device_sm_count());
+  const size_t need = tree_attn_ws_bytes(D, B, Hkv, mtiles, plan.splits);
   if (need > 0 && (ws == nullptr || ws_bytes < need || !aligned16(ws))) return TG_ERR_INVALID_ARG;
   a.ws = ws;
-  return launch_tree_attn(tq, tk, tv, a, splits, static_cast<cudaStream_t>(stream)) == cudaSuccess
+  a.coop = plan.coop;
+  return launch_tree_attn(tq, tk, tv, a, plan, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? TG_OK
              : TG_ERR_CUDA;
 }

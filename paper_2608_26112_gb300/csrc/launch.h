@@ -16,15 +16,24 @@ struct AttnArgs {
   float scale_log2;  // softmax scale * log2(e)
   void* out;
   float* lse_out;
-  void* ws;  // split-combine partial rows (tree_attn_ws_bytes)
+  void* ws;  // split counters + combine partial rows (tree_attn_ws_bytes)
   int* status;
+  int coop;  // 1: cooperative launch, split barrier on counters in ws; 0: clusters
+};
+// How one launch splits the keys: `splits` CTAs per work item, joined by a
+// thread-block cluster or, with coop, by a cooperative launch whose whole
+// grid is resident at once.
+struct AttnPlan {
+  int splits;
+  int coop;
 };
 // tmaps: q [D, Hq, n_total], k and v [D, B*Hkv*S_max] (innermost first)
 cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
-                             const CUtensorMap& tm_v, const AttnArgs& a, int kv_splits,
+                             const CUtensorMap& tm_v, const AttnArgs& a, AttnPlan plan,
                              cudaStream_t s);
-int tree_attn_pick_splits(int D, int B, int Hkv, int mtiles, int S_max, int num_sms);
+AttnPlan tree_attn_plan(int D, int B, int Hkv, int mtiles, int S_max, int num_sms);
 size_t tree_attn_ws_bytes(int D, int B, int Hkv, int mtiles, int splits);
+constexpr int kAttnMaxSplits = 10;
 
 struct TopkArgs {
   const void* logits;

@@ -46,7 +46,7 @@ constexpr int kSoftmaxThreads = 256;
 constexpr int kThreads = 64 + kSoftmaxThreads;
 constexpr int kAncWords = 9;  // 256 tree slots + one zero word
 constexpr int kRegion = 128 * 128;  // 128 rows x 128 bytes: one swizzled operand region
-constexpr int kMaxSplits = 8;
+constexpr int kClusterMaxSplits = 8;  // portable cluster size
 constexpr float kLn2 = 0.6931471805599453f;
 
 // K and V have their own rings: a K stage is free once its S = Q K^T
@@ -79,15 +79,14 @@ struct Layout {
   // consecutive rows) writes and reads 512 contiguous bytes: O as
   // [D / 4][kBM] float4 (column group major), then m[kBM] (base 2) and
   // l[kBM], then kBM * 2 spare floats.
-  static constexpr int kSlabFloats = kBM * (D + 4);
-  static constexpr int kSlabBytes = kSlabFloats * 4;
-  static constexpr int kSlabM = kBM * D;        // float offset of m[]
-  static constexpr int kSlabL = kBM * (D + 1);  // float offset of l[]
+  static constexpr int kSlabBytes = kBM * (2 * D + 8);
+  static constexpr int kSlabM = kBM * D * 2;  // byte offset of m[] (fp32)
+  static constexpr int kSlabL = kSlabM + kBM * 4;  // byte offset of l[] (fp32)
   static_assert(kAlloc <= 227 * 1024, "shared memory budget");
   static_assert(kOffQ % 1024 == 0 && kOffK % 1024 == 0 && kOffV % 1024 == 0 && kOffP % 1024 == 0,
                 "128-byte-swizzled operand tiles need 1024-byte alignment");
   static_assert(kOffBar % 8 == 0 && kOffMisc % 16 == 0, "mbarrier / scalar alignment");
-  static_assert(kSlabBytes % 16 == 0, "float4 slab");
+  static_assert(kSlabBytes % 16 == 0 && kSlabM % 16 == 0, "16-byte slab groups");
 };
 
 // 32 mask bits of one node for tree slots [b0, b0 + 32): slot < 0 is the
@@ -121,27 +120,47 @@ __device__ __forceinline__ void softmax_bar() {
   asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
 }
 
+// Workspace: two int counters per work item (the cooperative split
+// barrier), padded to 256 bytes, then the partial-row slabs.
+__host__ __device__ constexpr size_t attn_counter_bytes(long long units) {
+  return (size_t)((units * 8 + 255) / 256 * 256);
+}
+__device__ __forceinline__ float* attn_slabs(void* ws, long long units) {
+  return reinterpret_cast<float*>(static_cast<char*>(ws) + attn_counter_bytes(units));
+}
+__device__ __forceinline__ void red_add_release_gpu(int* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 // Columns one combine item covers with S splits: wide enough that a single
 // pass of the CTA's threads covers the rows it owns (ceil(128 / S) rows of
-// D columns), narrow enough that the S x COLS loaded floats stay in
+// D columns), narrow enough that the S x COLS loaded bf16 values stay in
 // registers, so every load of an item is in flight at once.
 template <int S>
 constexpr int combine_cols() {
-  return S <= 3 ? 32 : (S <= 6 ? 16 : 8);
+  return S <= 3 ? 64 : (S <= 6 ? 32 : 16);
 }
+static_assert(kAttnMaxSplits == 10, "combine_rows is instantiated for 2..10 splits");
 
 // Merge the S partial rows of the rows this CTA owns (Sec. 3.1 attention as
-// a softmax over the union of the splits' keys): o = sum_s w_s O_s / sum_s
-// w_s l_s with w_s = 2^(m_s - max_s m_s), lse = ln 2 (max + log2 sum).
+// a softmax over the union of the splits' keys).  Split s holds O_s / l_s
+// (bf16), its max m_s (base 2) and sum l_s: with w_s = 2^(m_s - M) l_s,
+// M = max_s m_s, the row is o = sum_s w_s (O_s / l_s) / sum_s w_s and
+// lse = ln 2 (M + log2 sum_s w_s).
 template <int D, int S>
-__device__ __forceinline__ void combine_rows(const float* slabs, int split, int r0, int G, int n,
+__device__ __forceinline__ void combine_rows(const char* slabs, int split, int r0, int G, int n,
                                              int off, int h, const AttnArgs& a) {
   using L = Layout<D>;
   constexpr int COLS = combine_cols<S>() < D ? combine_cols<S>() : D;
-  constexpr int NV = COLS / 4;  // float4 per split per item
+  constexpr int NV = COLS / 8;  // groups of 8 bf16 per split per item
   constexpr int CG = D / COLS;
   const float NEG_INF = __int_as_float(0xff800000);
-  const int rpc = (kBM + S - 1) / S;  // tile rows owned by each CTA of the cluster
+  const int rpc = (kBM + S - 1) / S;  // tile rows owned by each CTA of the work item
   const int row_lo = split * rpc;
   const int my_rows = max(0, min(kBM, row_lo + rpc) - row_lo);
   // items run row-fastest so that a warp reads consecutive rows of one
@@ -152,15 +171,15 @@ __device__ __forceinline__ void combine_rows(const float* slabs, int split, int 
     const int uu = rg / G, g = rg % G;
     if (uu >= n) continue;
     float mv[S], lv[S];
-    float4 ov[S][NV];
+    uint4 ov[S][NV];
 #pragma unroll
     for (int sp = 0; sp < S; ++sp) {
-      const float* src = slabs + (size_t)sp * L::kSlabFloats;
-      const float4* src4 = reinterpret_cast<const float4*>(src);
-      mv[sp] = __ldcg(src + L::kSlabM + rr);
-      lv[sp] = __ldcg(src + L::kSlabL + rr);
+      const char* src = slabs + (size_t)sp * L::kSlabBytes;
+      const uint4* src8 = reinterpret_cast<const uint4*>(src);
+      mv[sp] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabM) + rr);
+      lv[sp] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabL) + rr);
 #pragma unroll
-      for (int q = 0; q < NV; ++q) ov[sp][q] = __ldcg(src4 + (cg * NV + q) * kBM + rr);
+      for (int q = 0; q < NV; ++q) ov[sp][q] = __ldcg(src8 + (cg * NV + q) * kBM + rr);
     }
     float M = NEG_INF;
 #pragma unroll
@@ -171,21 +190,23 @@ __device__ __forceinline__ void combine_rows(const float* slabs, int split, int 
     for (int q = 0; q < COLS; ++q) acc[q] = 0.f;
 #pragma unroll
     for (int sp = 0; sp < S; ++sp) {
-      const float w = (mv[sp] == NEG_INF) ? 0.f : ex2(mv[sp] - M);
-      Ls += w * lv[sp];
+      const float w = (mv[sp] == NEG_INF) ? 0.f : ex2(mv[sp] - M) * lv[sp];
+      Ls += w;
 #pragma unroll
       for (int q = 0; q < NV; ++q) {
-        acc[4 * q + 0] += w * ov[sp][q].x;
-        acc[4 * q + 1] += w * ov[sp][q].y;
-        acc[4 * q + 2] += w * ov[sp][q].z;
-        acc[4 * q + 3] += w * ov[sp][q].w;
+        const uint32_t wd[4] = {ov[sp][q].x, ov[sp][q].y, ov[sp][q].z, ov[sp][q].w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          acc[8 * q + 2 * j] += w * __uint_as_float(wd[j] << 16);
+          acc[8 * q + 2 * j + 1] += w * __uint_as_float(wd[j] & 0xFFFF0000u);
+        }
       }
     }
     const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
     const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
     uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + cg * COLS);
 #pragma unroll
-    for (int q = 0; q < COLS / 8; ++q)
+    for (int q = 0; q < NV; ++q)
       dst[q] = make_uint4(pack_bf16(acc[8 * q + 0] * inv, acc[8 * q + 1] * inv),
                           pack_bf16(acc[8 * q + 2] * inv, acc[8 * q + 3] * inv),
                           pack_bf16(acc[8 * q + 4] * inv, acc[8 * q + 5] * inv),
@@ -205,8 +226,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   cg::cluster_group cluster = cg::this_cluster();
-  const int S_kv = (int)cluster.num_blocks();
-  const int split = (int)cluster.block_rank();
+  // the S_kv CTAs of a work item: a cluster, or (cooperative launch) the
+  // gridDim.x CTAs along x
+  const int S_kv = a.coop ? (int)gridDim.x : (int)cluster.num_blocks();
+  const int split = a.coop ? (int)blockIdx.x : (int)cluster.block_rank();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = a.Hq / a.Hkv;
   const int b = blockIdx.z / a.Hkv, h = blockIdx.z % a.Hkv;
@@ -559,11 +582,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (half == 0 && uu < n && a.lse_out)
         a.lse_out[orow] = live ? (m_run * sl2 + log2f(l_tot)) * kLn2 : NEG_INF;
     } else {
-      // ---- this row's partial straight into the workspace:
-      //      [O (D fp32) | m (base 2) | l | pad], read back after the cluster barrier
+      // ---- this row's partial straight into the workspace, read back
+      //      after the split barrier: O / l as bf16 plus (m base 2, l) in
+      //      fp32.  Rows past the tree's last node are never read.
       const size_t unit = (size_t)blockIdx.z * gridDim.y + blockIdx.y;
-      float* slab = reinterpret_cast<float*>(a.ws) + (unit * (size_t)S_kv + (size_t)split) * L::kSlabFloats;
-      float4* slab4 = reinterpret_cast<float4*>(slab);
+      char* slab = reinterpret_cast<char*>(attn_slabs(a.ws, gridDim.y * gridDim.z)) +
+                   (unit * (size_t)S_kv + (size_t)split) * L::kSlabBytes;
+      uint4* slab8 = reinterpret_cast<uint4*>(slab);  // [D / 8][kBM] groups of 8 bf16
+      const bool store = u < n;
+      const float inv = (live && l_tot > 0.f) ? 1.f / l_tot : 0.f;
       // tcgen05.ld / wait::ld are warp-collective: the condition must be the
       // same for the 32 lanes (ok and nt are); per-row liveness only selects
       // what is stored
@@ -573,19 +600,23 @@ __global__ void __launch_bounds__(kThreads, 1)
           float o[32];
           tmem_ld32f(tmem_O + lane_off + half * DH + c * 32, o);
           tc_wait_ld();
+          if (store) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            __stcg(slab4 + ((half * DH + c * 32) / 4 + q) * kBM + r,
-                   live ? make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3])
-                        : make_float4(0.f, 0.f, 0.f, 0.f));
+            for (int q = 0; q < 4; ++q)
+              __stcg(slab8 + ((half * DH + c * 32) / 8 + q) * kBM + r,
+                     make_uint4(pack_bf16(o[8 * q + 0] * inv, o[8 * q + 1] * inv),
+                                pack_bf16(o[8 * q + 2] * inv, o[8 * q + 3] * inv),
+                                pack_bf16(o[8 * q + 4] * inv, o[8 * q + 5] * inv),
+                                pack_bf16(o[8 * q + 6] * inv, o[8 * q + 7] * inv)));
+          }
         }
-      } else {
-        for (int c4 = 0; c4 < DH / 4; ++c4)
-          __stcg(slab4 + (half * DH / 4 + c4) * kBM + r, make_float4(0.f, 0.f, 0.f, 0.f));
+      } else if (store) {
+        for (int c8 = 0; c8 < DH / 8; ++c8)
+          __stcg(slab8 + (half * DH / 8 + c8) * kBM + r, make_uint4(0u, 0u, 0u, 0u));
       }
-      if (half == 0) {
-        __stcg(slab + L::kSlabM + r, live ? m_run * sl2 : NEG_INF);
-        __stcg(slab + L::kSlabL + r, live ? l_tot : 0.f);
+      if (half == 0 && store) {
+        __stcg(reinterpret_cast<float*>(slab + L::kSlabM) + r, live ? m_run * sl2 : NEG_INF);
+        __stcg(reinterpret_cast<float*>(slab + L::kSlabL) + r, live ? l_tot : 0.f);
       }
     }
   }
@@ -599,16 +630,46 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
 
-  // ---- combine through L2: every CTA has written its partial rows; the
+  // ---- combine through L2: every CTA has written its partial rows.  The
   // cluster barrier (release / acquire at cluster scope) makes them visible
-  // to the other CTAs of the cluster, and ends this CTA's TMEM reads
-  cluster.sync();
+  // to the other CTAs of the cluster.  In a cooperative launch the CTAs of
+  // a work item meet on a counter instead: thread 0 adds with release
+  // semantics (after the block barrier, so it covers every thread's
+  // stores) and waits, bounded, until all S_kv have arrived (acquire).
+  const size_t unit = (size_t)blockIdx.z * gridDim.y + blockIdx.y;
+  if (a.coop) {
+    __syncthreads();
+    if (tid == 0) {
+      int* cnt = reinterpret_cast<int*>(a.ws) + 2 * unit;
+      red_add_release_gpu(cnt, 1);
+      const long long t0 = clock64();
+      bool ok = true;
+      while (ld_acquire_gpu(cnt) < S_kv) {
+        if (clock64() - t0 > kWaitBudgetCycles) {
+          ok = false;
+          break;
+        }
+        __nanosleep(64);
+      }
+      if (!ok) raise_status(a.status, kStTimeout);
+      // every CTA of the item has passed the wait once the second counter
+      // reaches S_kv: its last arrival returns both counters to zero for
+      // the next launch
+      if (atomicAdd(cnt + 1, 1) == S_kv - 1) {
+        atomicExch(cnt, 0);
+        atomicExch(cnt + 1, 0);
+      }
+    }
+    __syncthreads();
+  } else {
+    cluster.sync();
+  }
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
-  const size_t unit = (size_t)blockIdx.z * gridDim.y + blockIdx.y;
-  const float* slabs = reinterpret_cast<const float*>(a.ws) + unit * (size_t)S_kv * L::kSlabFloats;
+  const char* slabs = reinterpret_cast<const char*>(attn_slabs(a.ws, gridDim.y * gridDim.z)) +
+                      unit * (size_t)S_kv * L::kSlabBytes;
   switch (S_kv) {
     case 2: combine_rows<D, 2>(slabs, split, r0, G, n, off, h, a); break;
     case 3: combine_rows<D, 3>(slabs, split, r0, G, n, off, h, a); break;
@@ -616,13 +677,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     case 5: combine_rows<D, 5>(slabs, split, r0, G, n, off, h, a); break;
     case 6: combine_rows<D, 6>(slabs, split, r0, G, n, off, h, a); break;
     case 7: combine_rows<D, 7>(slabs, split, r0, G, n, off, h, a); break;
-    default: combine_rows<D, 8>(slabs, split, r0, G, n, off, h, a); break;
+    case 8: combine_rows<D, 8>(slabs, split, r0, G, n, off, h, a); break;
+    case 9: combine_rows<D, 9>(slabs, split, r0, G, n, off, h, a); break;
+    default: combine_rows<D, 10>(slabs, split, r0, G, n, off, h, a); break;
   }
 }
 
 template <int D>
 cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                     const AttnArgs& a, int splits, cudaStream_t s) {
+                     const AttnArgs& a, AttnPlan plan, cudaStream_t s) {
   using L = Layout<D>;
   auto kern = tree_attn_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc);
@@ -630,15 +693,20 @@ cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtenso
   const int G = a.Hq / a.Hkv;
   const int mtiles = (G * a.max_nodes + kBM - 1) / kBM;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(splits, mtiles, a.B * a.Hkv);
+  cfg.gridDim = dim3(plan.splits, mtiles, a.B * a.Hkv);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = L::kAlloc;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = splits;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
+  if (plan.coop) {
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+  } else {
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = plan.splits;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+  }
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, tq, tk, tv, a);
@@ -671,52 +739,80 @@ int max_active_clusters_d(int splits) {
   return n;
 }
 
+// CTAs of this kernel resident on one SM
+template <int D>
+int blocks_per_sm_d() {
+  using L = Layout<D>;
+  auto kern = tree_attn_kernel<D>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc) !=
+      cudaSuccess)
+    return 0;
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, kThreads, L::kAlloc) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
 }  // namespace
 
-// KV splits per work item.  Cost model: waves of resident clusters times the
-// per-CTA time, a fixed part plus one part per 128-key tile of its split.
-// The number of clusters that fit at once comes from the occupancy API
-// (cached per device, head size and split count).
-int tree_attn_pick_splits(int D, int B, int Hkv, int mtiles, int S_max, int num_sms) {
-  static int cache[64][2][kMaxSplits + 1] = {};
+// How to split the keys.  Cost model: waves of resident work items times
+// the per-CTA time, a fixed part plus one part per 128-key tile of its
+// split.  A cluster path holds up to 8 splits, with the resident clusters
+// per split count from the occupancy API; a cooperative path holds up to
+// kAttnMaxSplits when the whole grid is resident at once (one wave).  On a
+// tie the cluster path wins (no counters).  Occupancy figures are cached
+// per device and head size.
+AttnPlan tree_attn_plan(int D, int B, int Hkv, int mtiles, int S_max, int num_sms) {
+  static int cache[64][2][kClusterMaxSplits + 1] = {};
+  static int bps_cache[64][2] = {};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
   const int di = D == 64 ? 0 : 1;
   const long long units = (long long)B * Hkv * mtiles;
   const int tiles = (S_max + kBN - 1) / kBN;
   const double kFixed = 5.0, kCombine = 1.0, kPerTile = 0.9;  // microseconds, measured scale
-  int best = 1;
+  int& bps = bps_cache[dev][di];
+  if (bps == 0) bps = di ? blocks_per_sm_d<128>() : blocks_per_sm_d<64>();
+  const long long coop_cap = (long long)(bps > 0 ? bps : 1) * num_sms;
+  AttnPlan best{1, 0};
   double best_cost = 1e30;
-  for (int s = 1; s <= kMaxSplits; ++s) {
+  for (int s = 1; s <= kAttnMaxSplits; ++s) {
     if (s > 1 && s > tiles) break;
-    int& fit = cache[dev][di][s];
-    if (fit == 0) fit = di ? max_active_clusters_d<128>(s) : max_active_clusters_d<64>(s);
-    const int resident = fit > 0 ? fit : (s == 1 ? num_sms : num_sms / (2 * s));
-    if (resident <= 0) continue;
-    const long long waves = (units + resident - 1) / resident;
-    const double cost = (double)waves * (kFixed + (s > 1 ? kCombine : 0.0) +
-                                         kPerTile * (double)((tiles + s - 1) / s));
-    if (cost < best_cost - 1e-9) {
-      best_cost = cost;
-      best = s;
+    const double per_cta = kFixed + (s > 1 ? kCombine : 0.0) + kPerTile * (double)((tiles + s - 1) / s);
+    if (s <= kClusterMaxSplits) {
+      int& fit = cache[dev][di][s];
+      if (fit == 0) fit = di ? max_active_clusters_d<128>(s) : max_active_clusters_d<64>(s);
+      const int resident = fit > 0 ? fit : (s == 1 ? num_sms : num_sms / (2 * s));
+      if (resident > 0) {
+        const double cost = (double)((units + resident - 1) / resident) * per_cta;
+        if (cost < best_cost - 1e-9) {
+          best_cost = cost;
+          best = AttnPlan{s, 0};
+        }
+      }
+    }
+    if (s > 1 && units * s <= coop_cap && per_cta < best_cost - 1e-9) {
+      best_cost = per_cta;
+      best = AttnPlan{s, 1};
     }
   }
   return best;
 }
 
-
-
 size_t tree_attn_ws_bytes(int D, int B, int Hkv, int mtiles, int splits) {
   if (splits <= 1) return 0;
   const size_t slab = D == 64 ? (size_t)Layout<64>::kSlabBytes : (size_t)Layout<128>::kSlabBytes;
-  return (size_t)B * Hkv * mtiles * splits * slab;
+  const long long units = (long long)B * Hkv * mtiles;
+  return attn_counter_bytes(units) + (size_t)units * splits * slab;
 }
 
 cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
-                             const CUtensorMap& tm_v, const AttnArgs& a, int kv_splits,
+                             const CUtensorMap& tm_v, const AttnArgs& a, AttnPlan plan,
                              cudaStream_t s) {
-  if (a.D == 64) return launch_d<64>(tm_q, tm_k, tm_v, a, kv_splits, s);
-  return launch_d<128>(tm_q, tm_k, tm_v, a, kv_splits, s);
+  if (a.D == 64) return launch_d<64>(tm_q, tm_k, tm_v, a, plan, s);
+  return launch_d<128>(tm_q, tm_k, tm_v, a, plan, s);
 }
 
 }  // namespace tg

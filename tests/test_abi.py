@@ -43,8 +43,10 @@ def test_status_strings(lib):
 
 
 def test_tree_attn_workspace_size(lib):
-    # one fp32 slab of 128 rows x (D + 4) floats per (tree, kv-head, row tile, split), 8 splits
-    assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 128) == 1 * 8 * 2 * 8 * 128 * 132 * 4
+    # two int counters per (tree, kv-head, row tile) padded to 256 bytes, then per
+    # (tree, kv-head, row tile, split) a slab of 128 rows x (D bf16 + 2 fp32), up to 10 splits
+    units = 1 * 8 * 2
+    assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 128) == 256 + units * 10 * 128 * 264
     assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 96) == 0
 
 
