@@ -11,8 +11,8 @@ decodes them itself.
 Every function is pinned against something other than itself by the
 CPU-only tests in tests/test_oracle_pins.py (brute force, closed forms,
 invariants).  Parity status per function:
-  ancestor_mask, tree_attention, expand_topk, rescore_select, accept:
-  pinned.
+  ancestor_mask, tree_attention, expand_topk, rescore_select, accept,
+  global_prune: pinned.
 
 Readings of the paper taken here (where it is silent or loose):
   * depth(root) = 0; mask row u has P + depth(u) + 1 ones (Algorithm 3 mask:
@@ -28,7 +28,9 @@ Readings of the paper taken here (where it is silent or loose):
   * verification at temperature 0 is greedy matching against the target's
     argmax (lowest token on ties); the accepted node is the deepest fully
     matching node, ties to the lowest id; the bonus token is the argmax of
-    the accepted node's own row.
+    the accepted node's own row;
+  * GlobalPrune (Algorithm 3) re-indexes the kept nodes in their original
+    order and lists retrieval paths by leaf in ascending new index.
 """
 from __future__ import annotations
 
@@ -252,3 +254,79 @@ def accept(target_logits, token, parent, node_off, path_cap: int, *, bf16: bool 
         alen[b] = len(chain) - 1
         bonus[b] = am[chain[-1]]
     return path, alen, bonus
+
+
+def global_prune(parent, score, node_off, budget: int, path_cap: int):
+    """Global score-based pruning with ancestor closure (Algorithm 3), per
+    tree, with the verification buffers it returns.
+
+    M = budget + 1 (the root is the extra node).  A tree with at most M
+    nodes is returned unchanged.  Otherwise the non-root nodes are ranked by
+    (-s(v), d(v), id(v)); starting from K = {root}, each ranked node's chain
+    up to the first node already in K is added whole when |K| + |chain| <= M,
+    and the loop stops once |K| = M.  The kept nodes are re-indexed in their
+    original order (parents keep coming before children), the mask is the
+    Algorithm 3 mask of the pruned tree, a node's position id is its depth,
+    and the retrieval paths are the root-to-leaf paths of the pruned tree
+    (leaves in ascending new index, root first, -1 padded to path_cap).
+    Scores are log-domain path scores (larger is better) in fp32.
+
+    Returns per tree b (arrays of stride Mo = min(M, max tree size)):
+      kept int32 [B, Mo] (old local ids in new order, -1 padded),
+      n_kept int32 [B], new_parent int32 [B, Mo] (-1 for the root and pad),
+      position int32 [B, Mo] (-1 pad), mask bool [B, Mo, Mo],
+      paths int32 [B, Mo, path_cap] (-1 padded), n_paths int32 [B].
+    """
+    slices = _tree_slices(node_off)
+    M = budget + 1
+    Mo = min(M, max(e - a for a, e in slices))
+    B = len(slices)
+    kept_o = np.full((B, Mo), -1, dtype=np.int32)
+    n_kept = np.zeros(B, dtype=np.int32)
+    par_o = np.full((B, Mo), -1, dtype=np.int32)
+    pos_o = np.full((B, Mo), -1, dtype=np.int32)
+    mask_o = np.zeros((B, Mo, Mo), dtype=bool)
+    paths_o = np.full((B, Mo, path_cap), -1, dtype=np.int32)
+    n_paths = np.zeros(B, dtype=np.int32)
+    for b, (a, e) in enumerate(slices):
+        par = [int(x) for x in parent[a:e]]
+        s = [float(x) for x in np.asarray(score[a:e], dtype=np.float32)]
+        check_tree(np.asarray(par))
+        n = e - a
+        d = node_depth(np.asarray(par))
+        if n <= M:
+            kept = list(range(n))
+        else:
+            ranked = sorted(range(1, n), key=lambda v: (-s[v], int(d[v]), v))
+            K = {0}
+            for v in ranked:
+                chain = []
+                w = v
+                while w not in K:
+                    chain.append(w)
+                    w = par[w]
+                if len(K) + len(chain) <= M:
+                    K.update(chain)
+                if len(K) == M:
+                    break
+            kept = sorted(K)
+        new = {old: i for i, old in enumerate(kept)}
+        new_par = [-1] + [new[par[v]] for v in kept[1:]]
+        k = len(kept)
+        n_kept[b] = k
+        kept_o[b, :k] = kept
+        par_o[b, :k] = new_par
+        pos_o[b, :k] = [int(d[v]) for v in kept]
+        mask_o[b, :k, :k] = ancestor_mask(np.asarray(new_par))
+        has_child = set(new_par[1:])
+        leaves = [i for i in range(k) if i not in has_child]
+        for j, leaf in enumerate(leaves):
+            chain = [leaf]
+            while new_par[chain[-1]] != -1:
+                chain.append(new_par[chain[-1]])
+            chain.reverse()
+            if len(chain) > path_cap:
+                raise ValueError("retrieval path longer than path_cap")
+            paths_o[b, j, :len(chain)] = chain
+        n_paths[b] = len(leaves)
+    return kept_o, n_kept, par_o, pos_o, mask_o, paths_o, n_paths

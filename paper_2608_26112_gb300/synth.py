@@ -107,6 +107,37 @@ def sample_tree(rng, n: int, depth: int, cap: int | None = None,
     return np.asarray(parent, dtype=np.int32)
 
 
+def expansion_tree(rng, D: int, W: int, m: int) -> np.ndarray:
+    """Parent array with the shape of a tree grown by D expansion steps of
+    frontier W and branching m (Algorithm 1's shape before pruning): the
+    root gets m children; at every later step W nodes of the newest level
+    (drawn at random here) get m children each.  Ids run level by level,
+    children grouped by parent, so parent[i] < i."""
+    parent = [-1]
+    level = [0]
+    for k in range(D):
+        front = level if k == 0 else sorted(rng.choice(level, size=min(W, len(level)), replace=False).tolist())
+        nxt = []
+        for v in front:
+            for _ in range(m):
+                parent.append(int(v))
+                nxt.append(len(parent) - 1)
+        level = nxt
+    return np.asarray(parent, dtype=np.int32)
+
+
+def path_scores(rng, parent: np.ndarray, step: float = 0.5, levels: int = 4) -> np.ndarray:
+    """fp32 scores that never increase from a node to its children, as
+    sums of log-probabilities along a path are: s(root) = 0 and
+    s(v) = s(parent) - step * j with j uniform in {0, .., levels - 1}
+    (zero steps give exact ties between a node and its child)."""
+    s = np.zeros(len(parent), dtype=np.float64)
+    drop = rng.integers(0, levels, size=len(parent)) * step
+    for v in range(1, len(parent)):
+        s[v] = s[parent[v]] - drop[v]
+    return s.astype(np.float32)
+
+
 def sample_tokens(rng, n: int, V: int) -> np.ndarray:
     return rng.integers(0, V, size=n, dtype=np.int64).astype(np.int32)
 

@@ -461,3 +461,134 @@ def test_accept_batched_trees_are_independent():
     for b in range(3):
         p1, a1, b1 = O.accept(x[off[b]:off[b + 1]], tok[off[b]:off[b + 1]], parents[b], [0, ns[b]], 8)
         assert np.array_equal(path[b], p1[0]) and A[b] == a1[0] and bonus[b] == b1[0]
+
+
+# ------------------------------------------------------------------ GlobalPrune (Algorithm 3)
+
+def top_nodes(parent, score, M):
+    """Root plus the M - 1 best non-root nodes by (score desc, depth asc,
+    id asc), by a library sort."""
+    n = len(parent)
+    d = O.node_depth(parent)
+    ids = np.arange(1, n)
+    order = np.lexsort((ids, d[1:], -np.asarray(score, np.float64)[1:]))
+    return sorted([0] + ids[order[:M - 1]].tolist())
+
+
+def check_prune_buffers(parent, kept, k, new_par, pos, mask, paths, n_paths):
+    """Properties any GlobalPrune result must have."""
+    kept = kept[:k].tolist()
+    assert kept[0] == 0 and kept == sorted(kept)
+    ks = set(kept)
+    for v in kept[1:]:
+        assert int(parent[v]) in ks                          # ancestor-closed
+    d = O.node_depth(parent)
+    for i, v in enumerate(kept):
+        assert pos[i] == d[v]
+        assert new_par[i] == (-1 if i == 0 else kept.index(int(parent[v])))
+    np.testing.assert_array_equal(mask[:k, :k], O.ancestor_mask(new_par[:k]))
+    assert not mask[k:].any() and not mask[:, k:].any()
+    leaves = [i for i in range(k) if i not in set(new_par[1:k].tolist())]
+    assert n_paths == len(leaves)
+    for j, leaf in enumerate(leaves):
+        row = paths[j]
+        length = int((row >= 0).sum())
+        assert row[length - 1] == leaf and row[0] == 0
+        assert all(new_par[row[t]] == row[t - 1] for t in range(1, length))
+        assert (row[length:] == -1).all()
+    assert (paths[n_paths:] == -1).all()
+
+
+def test_global_prune_small_tree_is_returned_unchanged():
+    rng = synth.make_rng(60)
+    parent = synth.sample_tree(rng, 12, 4)
+    score = synth.normal_f32(rng, (12,), 2.0)
+    kept, k, new_par, pos, mask, paths, npth = O.global_prune(parent, score, [0, 12], 11, 8)
+    assert k[0] == 12 and list(kept[0]) == list(range(12))
+    np.testing.assert_array_equal(new_par[0], parent)
+    np.testing.assert_array_equal(pos[0], O.node_depth(parent))
+    check_prune_buffers(parent, kept[0], 12, new_par[0], pos[0], mask[0], paths[0], npth[0])
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_global_prune_path_monotone_scores_keep_the_top_nodes(seed):
+    """With scores that never increase from parent to child (sums of
+    log-probabilities), every node ranks after its parent, each ranked chain
+    is the node alone, and Algorithm 3 keeps exactly the root and the
+    budget's best nodes."""
+    rng = synth.make_rng(61 + seed)
+    parent = synth.expansion_tree(rng, 5, 4, 3)
+    score = synth.path_scores(rng, parent)
+    n = len(parent)
+    for budget in (1, 7, 20, n - 2):
+        kept, k, new_par, pos, mask, paths, npth = O.global_prune(parent, score, [0, n], budget, 12)
+        assert kept[0, :k[0]].tolist() == top_nodes(parent, score, budget + 1)
+        check_prune_buffers(parent, kept[0], k[0], new_par[0], pos[0], mask[0], paths[0], npth[0])
+
+
+def test_global_prune_chain_keeps_the_first_nodes():
+    """On a chain every node's ancestors are the nodes before it, so only
+    chains ending at nodes 1..M-1 fit: the first M nodes are kept, whatever
+    the scores."""
+    rng = synth.make_rng(62)
+    n = 30
+    parent = np.arange(-1, n - 1, dtype=np.int32)
+    score = synth.normal_f32(rng, (n,), 5.0)
+    kept, k, new_par, pos, mask, paths, npth = O.global_prune(parent, score, [0, n], 9, 12)
+    assert kept[0, :k[0]].tolist() == list(range(10))
+    assert npth[0] == 1 and paths[0, 0].tolist() == list(range(10)) + [-1, -1]
+
+
+def test_global_prune_star_is_plain_top_k():
+    rng = synth.make_rng(63)
+    n = 40
+    parent = np.zeros(n, dtype=np.int32)
+    parent[0] = -1
+    score = np.round(synth.normal_f32(rng, (n,), 2.0)).astype(np.float32)  # many ties
+    kept, k, *_ = O.global_prune(parent, score, [0, n], 12, 3)
+    ids = np.arange(1, n)
+    order = np.lexsort((ids, -score[1:].astype(np.float64)))
+    assert kept[0, :k[0]].tolist() == sorted([0] + ids[order[:12]].tolist())
+
+
+def test_global_prune_skips_a_long_chain_and_keeps_ranking():
+    """Worked by hand from Algorithm 3 with M = 3: the best node x sits at
+    depth 3 and its chain (x, b, a) would make |K| = 4 > 3, so it is
+    skipped; c and e then fit and fill K = {r, c, e}."""
+    #          r   a  b  x  c  e
+    parent = np.array([-1, 0, 1, 2, 0, 0], np.int32)
+    score = np.array([0, -1, -2, 10, 5, 4], np.float32)
+    kept, k, new_par, pos, mask, paths, npth = O.global_prune(parent, score, [0, 6], 2, 3)
+    assert kept[0, :k[0]].tolist() == [0, 4, 5]
+    assert new_par[0].tolist() == [-1, 0, 0] and pos[0].tolist() == [0, 1, 1]
+    assert npth[0] == 2 and paths[0].tolist() == [[0, 1, -1], [0, 2, -1], [-1, -1, -1]]
+
+
+def test_global_prune_ties_prefer_shallower_then_lower_id():
+    """Equal scores: depth decides (shallower first), then the lower id."""
+    #          r  a  b  c  d
+    parent = np.array([-1, 0, 1, 0, 0], np.int32)
+    score = np.array([0, 1, 3, 3, 3], np.float32)      # b (depth 2) ties c, d (depth 1)
+    kept, k, *_ = O.global_prune(parent, score, [0, 5], 2, 4)
+    assert kept[0, :k[0]].tolist() == [0, 3, 4]        # c, d before b; b's chain no longer fits
+    kept, k, *_ = O.global_prune(parent, score, [0, 5], 1, 4)
+    assert kept[0, :k[0]].tolist() == [0, 3]           # c before d by id
+
+
+def test_global_prune_random_scores_batched_invariants():
+    rng = synth.make_rng(64)
+    parents, scores, off = [], [], [0]
+    for n in (1, 9, 40, 77):
+        p = synth.sample_tree(rng, n, min(n - 1, 6)) if n > 1 else np.array([-1], np.int32)
+        parents.append(p)
+        scores.append(synth.normal_f32(rng, (n,), 3.0))
+        off.append(off[-1] + n)
+    par, sc = np.concatenate(parents), np.concatenate(scores)
+    out = O.global_prune(par, sc, off, 15, 10)
+    for b in range(4):
+        single = O.global_prune(parents[b], scores[b], [0, len(parents[b])], 15, 10)
+        assert out[1][b] == single[1][0]
+        Mo = out[0].shape[1]
+        check_prune_buffers(parents[b], out[0][b], out[1][b], out[2][b], out[3][b], out[4][b],
+                            out[5][b], out[6][b])
+        assert out[1][b] <= 16
