@@ -185,6 +185,37 @@ def time_graph(g, reps, stream):
     return e0.elapsed_time(e1) / 1e3  # seconds
 
 
+def prune_timing(R, seed, dev, stream, reps):
+    """GlobalPrune (Algorithm 3) timed beside the step, not inside it: the
+    pre-pruning tree of the Llama-3-8B-shaped verify step (6 expansion steps
+    of frontier 10 and branching 10: 511 nodes) with path-sum scores,
+    pruned to a 59-node budget; R input sets, one launch each."""
+    import numpy as np
+    import torch
+    import paper_2608_26112_gb300 as tg
+    from paper_2608_26112_gb300 import synth
+
+    sets = []
+    for r in range(R):
+        rng = synth.make_rng(20_000 + seed + r)
+        par = synth.expansion_tree(rng, 6, 10, 10)
+        sc = synth.path_scores(rng, par)
+        sets.append((torch.from_numpy(sc).to(dev), torch.from_numpy(par).to(dev),
+                     torch.tensor([0, len(par)], dtype=torch.int32, device=dev), len(par)))
+    outs = []
+    with torch.cuda.stream(stream):
+        for sc, par, off, n in sets:
+            outs.append(tg.global_prune(sc, par, off, n, 59, 8, stream=stream))
+    stream.synchronize()
+    g = capture(lambda: [tg.global_prune(sc, par, off, n, 59, 8, out=o, stream=stream)
+                         for (sc, par, off, n), o in zip(sets, outs)], stream)
+    g.replay()
+    t = time_graph(g, reps, stream) / (reps * R)
+    n = sets[0][3]
+    return {"us": t * 1e6, "nodes_in": n, "budget": 59, "bytes": n * 8 + 60 * 16,
+            "in_step": False, "note": "Algorithm 3 on the pre-pruning tree, latency-bound"}
+
+
 # --------------------------------------------------------------------------- clocks
 
 class ClockSampler:
@@ -451,6 +482,7 @@ def ours_arm(args):
         for name, g in per_kernel_graphs.items():
             g.replay()
             kt[name] = time_graph(g, kreps, stream) / (kreps * R)
+        prune = prune_timing(R, rank_seed(args.seed, rank), dev, stream, kreps)
     assert tg.last_device_status(stream) == 0
     t_max = max_over_ranks(t_steps, world)
     steps_per_s = job_throughput(world, K, t_max)
@@ -465,6 +497,7 @@ def ours_arm(args):
                          "hbm_frac": b / kt[name] / 1e9 / hbm}
         if f:
             kernels[name]["TFLOPs"] = f / kt[name] / 1e12
+    kernels["global_prune"] = prune
     dom = max(KERNELS, key=lambda n: kt[n])
     b, f = costs[dom]
     achieved = b / kt[dom] / 1e9

@@ -237,6 +237,48 @@ int treegraft_accept_noalloc(const void* target_logits, int dtype, int V, int64_
                              void* stream);
 
 /*
+ * treegraft_global_prune - global score-based pruning with ancestor closure,
+ * and the verification buffers of the pruned tree.
+ *
+ * Paper: Algorithm 3 (GlobalPrune, called by Algorithms 1 and 2 before
+ * target verification).  Per tree, with M = budget + 1 (the root is the
+ * extra node): a tree of at most M nodes is kept whole; otherwise the
+ * non-root nodes are ranked by (score desc, depth asc, id asc) and, from
+ * K = {root}, each ranked node's chain up to the first node in K is added
+ * whole when |K| + |chain| <= M, stopping once |K| = M.  Kept nodes are
+ * re-indexed in their original order (parents stay before children).
+ *
+ * score    fp32 [n_total] path scores (log domain, larger is better; the
+ *          root's is ignored).  Finite or -inf.
+ * parent   int32 [n_total] local parent ids; node_off int32 [B+1]; trees of
+ *          1..TG_MAX_PRUNE_NODES nodes, n_total <= B * max_nodes.
+ * budget   B_ver >= 1 with budget + 1 <= TG_MAX_TREE_NODES (the pruned
+ *          tree must fit treegraft_tree_attn).
+ * Outputs, with stride Mo = min(budget + 1, max_nodes) per tree:
+ *   kept       int32 [B, Mo]  old local ids in new order, -1 padded;
+ *   n_kept     int32 [B];
+ *   new_parent int32 [B, Mo]  parent in new ids (-1 for the root and pad);
+ *   position   int32 [B, Mo]  position id = depth (-1 pad);
+ *   mask       uint32 [B, Mo, ceil(Mo / 32)]  row i bit j set iff new node
+ *              j is the root, an ancestor of i, or i itself (Algorithm 3
+ *              mask); rows past n_kept are zero;
+ *   paths      int32 [B, Mo, path_cap]  root-to-leaf retrieval paths in new
+ *              ids, one row per leaf in ascending new id, root first, -1
+ *              padded; rows past n_paths are -1;
+ *   n_paths    int32 [B].
+ * Errors: TG_ERR_INVALID_ARG, TG_ERR_UNSUPPORTED (max_nodes >
+ *   TG_MAX_PRUNE_NODES), TG_ERR_CUDA; a malformed tree sets
+ *   TG_ERR_DEVICE_TREE (its outputs left unwritten); a path longer than
+ *   path_cap sets TG_ERR_DEVICE_INDEX (the path is cut at path_cap).
+ */
+#define TG_MAX_PRUNE_NODES 1024
+int treegraft_global_prune(const float* score, const int32_t* parent, const int32_t* node_off,
+                           int B, int max_nodes, int n_total, int budget, int path_cap,
+                           int32_t* kept, int32_t* n_kept, int32_t* new_parent,
+                           int32_t* position, uint32_t* mask, int32_t* paths, int32_t* n_paths,
+                           void* stream);
+
+/*
  * treegraft_last_device_status - synchronise `stream`, return the OR of the
  * device status bits raised since the last call on the current device
  * (TG_OK if none), and clear them.  Returns TG_ERR_CUDA if the

@@ -20,6 +20,7 @@ TG_OK = 0
 TG_BF16, TG_F32 = 0, 1
 MAX_TREE_NODES = 256
 MAX_TOPK = 32
+MAX_PRUNE_NODES = 1024
 
 _lib = None
 
@@ -49,6 +50,8 @@ _SIGNATURES = {
                          _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_size, _c_vp],
     "treegraft_accept_noalloc": [_c_vp, _c_int, _c_int, _c_i64, _c_vp, _c_vp, _c_vp, _c_int,
                                  _c_int, _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp],
+    "treegraft_global_prune": [_c_vp, _c_vp, _c_vp, _c_int, _c_int, _c_int, _c_int, _c_int,
+                               _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp],
     "treegraft_last_device_status": [_c_vp],
     "treegraft_status_string": [_c_int],
 }
@@ -265,3 +268,34 @@ def accept_noalloc(target_logits, token, parent, node_off, max_nodes, path_cap, 
 def last_device_status(stream=None) -> int:
     """Synchronise the stream; return and clear the device status bits."""
     return int(lib().treegraft_last_device_status(_stream(stream)))
+
+
+def global_prune(score, parent, node_off, max_nodes, budget, path_cap, *, out=None, stream=None):
+    """GlobalPrune of each tree to budget + 1 nodes with its verification
+    buffers (Algorithm 3).  score fp32 [n_total], parent / node_off int32.
+    Returns (kept, n_kept, new_parent, position, mask, paths, n_paths) with
+    Mo = min(budget + 1, max_nodes) rows per tree; mask holds the uint32 bit
+    words as int32 [B, Mo, ceil(Mo / 32)]."""
+    _need(score, torch.float32, "score")
+    _need(parent, torch.int32, "parent")
+    _need(node_off, torch.int32, "node_off")
+    n_total = parent.shape[0]
+    B = node_off.shape[0] - 1
+    Mo = min(int(budget) + 1, int(max_nodes))
+    W = (Mo + 31) // 32
+    dev = parent.device
+    if out is None:
+        out = (torch.empty(B, Mo, dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev),
+               torch.empty(B, Mo, dtype=torch.int32, device=dev),
+               torch.empty(B, Mo, dtype=torch.int32, device=dev),
+               torch.empty(B, Mo, W, dtype=torch.int32, device=dev),
+               torch.empty(B, Mo, int(path_cap), dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev))
+    kept, n_kept, new_parent, position, mask, paths, n_paths = out
+    st = lib().treegraft_global_prune(_ptr(score), _ptr(parent), _ptr(node_off), B, int(max_nodes),
+                                      n_total, int(budget), int(path_cap), _ptr(kept),
+                                      _ptr(n_kept), _ptr(new_parent), _ptr(position), _ptr(mask),
+                                      _ptr(paths), _ptr(n_paths), _stream(stream))
+    _check("treegraft_global_prune", st)
+    return kept, n_kept, new_parent, position, mask, paths, n_paths

@@ -4,6 +4,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <mutex>
@@ -236,6 +237,41 @@ size_t treegraft_accept_workspace_size(int B, int n_total) {
   if (B < 1 || n_total < 1) return 0;
   const size_t bytes = ((size_t)n_total + (size_t)B) * sizeof(int32_t);
   return (bytes + 255) & ~(size_t)255;
+}
+
+int treegraft_global_prune(const float* score, const int32_t* parent, const int32_t* node_off,
+                           int B, int max_nodes, int n_total, int budget, int path_cap,
+                           int32_t* kept, int32_t* n_kept, int32_t* new_parent,
+                           int32_t* position, uint32_t* mask, int32_t* paths, int32_t* n_paths,
+                           void* stream) {
+  if (!score || !parent || !node_off || !kept || !n_kept || !new_parent || !position || !mask ||
+      !paths || !n_paths)
+    return TG_ERR_INVALID_ARG;
+  if (B < 1 || max_nodes < 1 || n_total < 1 || (long long)n_total > (long long)B * max_nodes ||
+      budget < 1 || budget + 1 > TG_MAX_TREE_NODES || path_cap < 1)
+    return TG_ERR_INVALID_ARG;
+  if (max_nodes > TG_MAX_PRUNE_NODES) return TG_ERR_UNSUPPORTED;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  PruneArgs a;
+  a.score = score;
+  a.parent = parent;
+  a.node_off = node_off;
+  a.B = B;
+  a.n_total = n_total;
+  a.budget = budget;
+  a.stride = std::min(budget + 1, max_nodes);
+  a.path_cap = path_cap;
+  a.kept = kept;
+  a.n_kept = n_kept;
+  a.new_parent = new_parent;
+  a.position = position;
+  a.mask = mask;
+  a.paths = paths;
+  a.n_paths = n_paths;
+  a.status = st;
+  return launch_global_prune(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK
+                                                                                 : TG_ERR_CUDA;
 }
 
 int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld, const int32_t* token,

@@ -89,6 +89,22 @@ struct AcceptArgs {
 };
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s);
 
+struct PruneArgs {
+  const float* score;
+  const int32_t* parent;
+  const int32_t* node_off;
+  int B, n_total, budget, stride, path_cap;
+  int32_t* kept;
+  int32_t* n_kept;
+  int32_t* new_parent;
+  int32_t* position;
+  uint32_t* mask;
+  int32_t* paths;
+  int32_t* n_paths;
+  int* status;
+};
+cudaError_t launch_global_prune(const PruneArgs& a, cudaStream_t s);
+
 int device_sm_count();
 // device address of the per-device status word (nullptr on failure)
 int* status_word_ptr();

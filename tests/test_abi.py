@@ -126,3 +126,17 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(binding, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="missing"):
         binding.lib()
+
+
+def test_global_prune_rejects_bad_args_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+
+    def call(B=1, max_nodes=100, n_total=100, budget=10, path_cap=8, score=fake):
+        return lib.treegraft_global_prune(score, fake, fake, B, max_nodes, n_total, budget,
+                                          path_cap, fake, fake, fake, fake, fake, fake, fake, NULL)
+    assert call(score=NULL) == 1
+    assert call(budget=0) == 1                   # empty verification budget
+    assert call(budget=256) == 1                 # pruned tree beyond tree_attn's 256 nodes
+    assert call(path_cap=0) == 1
+    assert call(n_total=101) == 1                # more nodes than B * max_nodes
+    assert call(max_nodes=2000, n_total=2000) == 2

@@ -460,3 +460,73 @@ def test_expand_topk_serving_rows(dev):
     got = _run_expand(_dev.bf16(lg, dev), ps, sh["k"], dev, row_idx=rows)
     ref = O.expand_topk(lg, ps, sh["k"], row_idx=rows, bf16=True)
     _check_expand(got, ref)
+
+
+
+# ------------------------------------------------------------------ GlobalPrune (Algorithm 3)
+
+def _mask_words(mask_bool):
+    """bool [B, Mo, Mo] -> uint32 words [B, Mo, ceil(Mo / 32)], bit j of word j // 32."""
+    B, Mo, _ = mask_bool.shape
+    W = (Mo + 31) // 32
+    out = np.zeros((B, Mo, W), dtype=np.uint32)
+    for j in range(Mo):
+        out[:, :, j // 32] |= mask_bool[:, :, j].astype(np.uint32) << np.uint32(j % 32)
+    return out
+
+
+def _run_prune(parents, scores, budget, path_cap, dev):
+    off = np.concatenate([[0], np.cumsum([len(p) for p in parents])]).astype(np.int32)
+    par, sc = np.concatenate(parents).astype(np.int32), np.concatenate(scores).astype(np.float32)
+    maxn = max(len(p) for p in parents)
+    got = tg.global_prune(_dev.f32(sc, dev), _dev.i32(par, dev), _dev.i32(off, dev), maxn, budget,
+                          path_cap)
+    _status_clean()
+    got = [t.cpu().numpy() for t in got]
+    got[4] = got[4].view(np.uint32)
+    ref = O.global_prune(par, sc, off, budget, path_cap)
+    return got, ref
+
+
+def _check_prune(got, ref):
+    kept, n_kept, new_par, pos, mask, paths, n_paths = got
+    rk, rn, rp, rpos, rmask, rpaths, rnp = ref
+    np.testing.assert_array_equal(n_kept, rn)
+    np.testing.assert_array_equal(kept, rk)
+    np.testing.assert_array_equal(new_par, rp)
+    np.testing.assert_array_equal(pos, rpos)
+    np.testing.assert_array_equal(mask, _mask_words(rmask))
+    np.testing.assert_array_equal(n_paths, rnp)
+    np.testing.assert_array_equal(paths, rpaths)
+
+
+@pytest.mark.parametrize("monotone", [True, False])
+def test_global_prune_expansion_trees(dev, monotone):
+    """Trees with the shape of 6 expansion steps of frontier 10 and branching
+    10 (511 nodes) and of smaller growths, pruned to a 59-node budget:
+    path-sum scores (the realistic case) and random scores (long chains)."""
+    rng = synth.make_rng(300 + monotone)
+    parents = [synth.expansion_tree(rng, 6, 10, 10), synth.expansion_tree(rng, 4, 3, 4),
+               synth.expansion_tree(rng, 3, 5, 8), synth.sample_tree(rng, 40, 5)]
+    scores = [synth.path_scores(rng, p) if monotone else synth.normal_f32(rng, (len(p),), 3.0)
+              for p in parents]
+    got, ref = _run_prune(parents, scores, 59, 12, dev)
+    _check_prune(got, ref)
+
+
+def test_global_prune_largest_trees_and_budgets(dev):
+    rng = synth.make_rng(310)
+    parents = [synth.sample_tree(rng, 1024, 9, 16), synth.sample_tree(rng, 700, 12),
+               np.array([-1], np.int32), synth.expansion_tree(rng, 5, 8, 8)]
+    scores = [synth.path_scores(rng, parents[0]), synth.normal_f32(rng, (700,), 2.0),
+              np.zeros(1, np.float32), np.round(synth.normal_f32(rng, (len(parents[3]),), 1.0))]
+    for budget in (1, 63, 255):
+        got, ref = _run_prune(parents, scores, budget, 16, dev)
+        _check_prune(got, ref)
+
+
+def test_global_prune_malformed_tree_sets_status(dev):
+    par = np.array([-1, 0, 3, 1], np.int32)            # parent after child
+    tg.global_prune(_dev.f32(np.zeros(4), dev), _dev.i32(par, dev), _dev.i32([0, 4], dev), 4, 2,
+                    4)
+    assert tg.last_device_status() & 4
