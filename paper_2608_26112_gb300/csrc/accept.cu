@@ -44,6 +44,8 @@ __global__ void __launch_bounds__(kScanThreads, 4) accept_kernel(AcceptArgs a, i
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int VW = ScanTraits<T>::kVW;
   const int V = a.V;
+  pdl_launch_dependents();
+  pdl_wait();
   cluster_arrive_relaxed();
   const int per = ((V + C - 1) / C + VW - 1) / VW * VW;
   const int c0 = min(V, crank * per);
@@ -178,13 +180,15 @@ cudaError_t launch_accept_t(const AcceptArgs& a, int C, cudaStream_t s) {
     cfg.gridDim = dim3(C, nr, 1);
     cfg.blockDim = dim3(kScanThreads, 1, 1);
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = C;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     cudaError_t e = cudaLaunchKernelEx(&cfg, kern, a, r0);
     if (e != cudaSuccess) return e;
   }

@@ -102,6 +102,18 @@ __device__ __forceinline__ void cluster_wait() {
   asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
 }
 
+// ---------------------------------------------------------------- dependent launch
+// Programmatic dependent launch.  pdl_wait blocks until the grid this one
+// depends on (the previous kernel on the stream) has completed and its
+// memory is visible - a no-op for a launch that did not opt in; it comes
+// before a kernel's first global-memory access, so the stream's order is
+// kept exactly.  pdl_launch_dependents lets the next kernel on the stream be
+// dispatched now, so its launch overlaps this kernel instead of following it.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- smem / mbarrier
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

@@ -63,6 +63,8 @@ __global__ void __launch_bounds__(kThreads, 1) global_prune_kernel(PruneArgs a) 
   __shared__ PruneSmem sm;
   const int b = blockIdx.x;
   const int v = threadIdx.x;
+  pdl_launch_dependents();
+  pdl_wait();
   const int off = a.node_off[b];
   const int n = a.node_off[b + 1] - off;
   const int M = a.budget + 1;
@@ -214,8 +216,16 @@ __global__ void __launch_bounds__(kThreads, 1) global_prune_kernel(PruneArgs a) 
 }  // namespace
 
 cudaError_t launch_global_prune(const PruneArgs& a, cudaStream_t s) {
-  global_prune_kernel<<<a.B, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.B, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, global_prune_kernel, a);
 }
 
 }  // namespace tg

@@ -28,6 +28,8 @@ __global__ void __launch_bounds__(kThreads) rescore_select_kernel(RescoreArgs a)
   __shared__ int red_i[8];
   const int b = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  pdl_launch_dependents();
+  pdl_wait();
   const int off = a.node_off[b];
   const int n = a.node_off[b + 1] - off;
   if (n < 1 || n > 256 || off < 0 || off + n > a.n_total) {
@@ -111,8 +113,16 @@ __global__ void __launch_bounds__(kThreads) rescore_select_kernel(RescoreArgs a)
 }  // namespace
 
 cudaError_t launch_rescore_select(const RescoreArgs& a, cudaStream_t s) {
-  rescore_select_kernel<<<a.B, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.B, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, rescore_select_kernel, a);
 }
 
 }  // namespace tg

@@ -78,6 +78,8 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   const int V = a.V;
   constexpr int VW = ScanTraits<T>::kVW;
 
+  pdl_launch_dependents();
+  pdl_wait();
   // physical row (uniform over the cluster: every CTA reads the same index)
   int r = row;
   if (a.row_idx) r = a.row_idx[row];
@@ -285,13 +287,15 @@ cudaError_t launch_topk_t(const TopkArgs& a, int C, cudaStream_t s) {
     cfg.blockDim = dim3(kScanThreads, 1, 1);
     cfg.dynamicSmemBytes = 0;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = C;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     cudaError_t e = cudaLaunchKernelEx(&cfg, kern, b);
     if (e != cudaSuccess) return e;
   }

@@ -249,6 +249,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t p_base = smem_u32(smem + L::kOffP);
   const float NEG_INF = __int_as_float(0xff800000);
 
+  // the next kernel on the stream may be dispatched now (it waits for this
+  // grid's completion before touching memory)
+  pdl_launch_dependents();
   // ---- the tree's extent (global reads in flight while the barriers are set up)
   const int off = a.node_off[b];
   const int n = a.node_off[b + 1] - off;
