@@ -12,7 +12,7 @@ Every function is pinned against something other than itself by the
 CPU-only tests in tests/test_oracle_pins.py (brute force, closed forms,
 invariants).  Parity status per function:
   ancestor_mask, tree_attention, expand_topk, rescore_select, accept,
-  global_prune: pinned.
+  global_prune, grow_tree: pinned.
 
 Readings of the paper taken here (where it is silent or loose):
   * depth(root) = 0; mask row u has P + depth(u) + 1 ones (Algorithm 3 mask:
@@ -330,3 +330,75 @@ def global_prune(parent, score, node_off, budget: int, path_cap: int):
             paths_o[b, j, :len(chain)] = chain
         n_paths[b] = len(leaves)
     return kept_o, n_kept, par_o, pos_o, mask_o, paths_o, n_paths
+
+
+def _row_log_softmax(logits, r: int, bf16: bool):
+    """(values, lse) of one logit row in fp64."""
+    x = _row_values(logits, r, bf16)
+    m = x.max()
+    lse = NEG_INF if m == NEG_INF else m + np.log(np.exp(x - m).sum())
+    return x, lse
+
+
+def grow_tree(schedule, W: int, m: int, small_logits, middle_logits, *, bf16: bool = False):
+    """TreeGraft shared-tree construction (Algorithm 2) for one sequence.
+
+    The drafters' next-token logits under the prefix ending at node v are
+    rows v of small_logits and middle_logits (tables indexed by node id, the
+    stand-in for the drafter forwards).  Scores are log-domain: s(root) = 0,
+    s(u) = fp32(s(v) + p(u)) with p(u) = fp32(l_u - lse) the drafter's
+    log-probability of u's token.  Step k with schedule[k] = 0 (small
+    drafter): C = N_k (the nodes made at the previous step; {root} at
+    first), F = Top_W(C, s) by (s desc, id asc), and each v in F gets its
+    m best small-drafter tokens (logit desc, token asc) as new children.
+    schedule[k] = 1 (middle drafter): C = V(T) \\ P; every non-root v in C is
+    rescored, p(v) = fp32(l_m[pa(v), token(v)] - lse_m[pa(v)]), and s is
+    recomputed in node order; F = Top_W(C, s); each v in F gets its m best
+    middle-drafter tokens; then P = P u C.  Children are appended in frontier
+    order, then child rank, never replacing an existing node.
+
+    Returns parent int32, token int32, edge f32, score f32 (per node), the
+    visited set P as uint8, and the list of frontiers (one per step).
+    """
+    parent, token = [-1], [0]
+    edge, score = [np.float32(0.0)], [np.float32(0.0)]
+    new = [0]
+    P = set()
+    lse_m = {}
+    frontiers = []
+    for a in schedule:
+        n = len(parent)
+        if a == 0:
+            C = list(new)
+            table = small_logits
+        else:
+            C = [v for v in range(n) if v not in P]
+            for v in C:
+                lse_m[v] = _row_log_softmax(middle_logits, v, bf16)[1]
+            for v in C:
+                if v == 0:
+                    continue
+                row = _row_values(middle_logits, parent[v], bf16)
+                edge[v] = np.float32(row[token[v]] - lse_m[parent[v]])
+                score[v] = np.float32(score[parent[v]] + edge[v])
+            table = middle_logits
+        F = sorted(C, key=lambda v: (-float(score[v]), v))[:W]
+        frontiers.append(F)
+        made = []
+        for v in F:
+            x, lse = _row_log_softmax(table, v, bf16)
+            order = np.lexsort((np.arange(len(x)), -x))[:m]
+            for y in order:
+                lp = np.float32(x[y] - lse)
+                parent.append(v)
+                token.append(int(y))
+                edge.append(lp)
+                score.append(np.float32(score[v] + lp))
+                made.append(len(parent) - 1)
+        if a == 1:
+            P.update(C)
+        new = made
+    visited = np.zeros(len(parent), dtype=np.uint8)
+    visited[sorted(P)] = 1
+    return (np.asarray(parent, np.int32), np.asarray(token, np.int32),
+            np.asarray(edge, np.float32), np.asarray(score, np.float32), visited, frontiers)

@@ -592,3 +592,98 @@ def test_global_prune_random_scores_batched_invariants():
         check_prune_buffers(parents[b], out[0][b], out[1][b], out[2][b], out[3][b], out[4][b],
                             out[5][b], out[6][b])
         assert out[1][b] <= 16
+
+
+# ------------------------------------------------------------------ grow loop (Algorithm 2)
+
+def _lsm(row):
+    from scipy.special import log_softmax
+    return log_softmax(np.asarray(row, np.float64))
+
+
+def test_grow_tree_hand_worked_graft():
+    """Worked by hand from Algorithm 2 with W = 1, m = 2 and schedule
+    (small, middle, small).  Step 1 expands the root with the small drafter's
+    two best tokens (1, 3).  Step 2: P is empty, so C = {r, 1, 2}; nodes 1
+    and 2 are rescored from the middle drafter's root row, the root (score
+    0, the largest possible) is the frontier and gets the middle drafter's
+    two best tokens 3 and 0 (tie at 0 to the lower token) - a second child
+    with token 3 is attached next to node 2, not over it.  Step 3 expands the
+    better of the new nodes {3, 4}: node 3."""
+    rng = synth.make_rng(70)
+    small = synth.normal_f32(rng, (8, 4), 1.0)
+    small[0] = [0.0, 3.0, 1.0, 2.0]
+    middle = synth.normal_f32(rng, (8, 4), 1.0)
+    middle[0] = [0.0, 0.0, 0.0, 5.0]
+    par, tok, edge, score, vis, fr = O.grow_tree([0, 1, 0], 1, 2, small, middle)
+    assert par.tolist() == [-1, 0, 0, 0, 0, 3, 3]
+    t56 = np.lexsort((np.arange(4), -small[3].astype(np.float64)))[:2].tolist()
+    assert tok.tolist() == [0, 1, 3, 3, 0] + t56
+    assert fr == [[0], [0], [3]]
+    assert vis.tolist() == [1, 1, 1, 0, 0, 0, 0]
+    lm, ls3 = _lsm(middle[0]), _lsm(small[3])
+    expect = [0.0, lm[1], lm[3], lm[3], lm[0], lm[3] + ls3[t56[0]], lm[3] + ls3[t56[1]]]
+    np.testing.assert_allclose(score, expect, atol=2e-6)
+    np.testing.assert_allclose(edge[1:3], [lm[1], lm[3]], atol=1e-6)   # rescored edges
+
+
+def test_grow_tree_all_small_is_single_drafter_construction():
+    """With every step on the small drafter, Algorithm 2 is Algorithm 1:
+    each frontier is the best W of the previous step's nodes, every node's
+    score is the sum of small-drafter log-probabilities along its path, and
+    nothing is visited."""
+    rng = synth.make_rng(71)
+    V, W, m, D = 32, 2, 3, 3
+    small = synth.normal_f32(rng, (64, V), 2.0)
+    middle = synth.normal_f32(rng, (64, V), 2.0)
+    par, tok, edge, score, vis, fr = O.grow_tree([0] * D, W, m, small, middle)
+    assert len(par) == 1 + m + W * m + W * m and not vis.any()
+    prev = [0]
+    for k in range(D):
+        best = sorted(prev, key=lambda v: (-float(score[v]), v))[:W]
+        assert fr[k] == best
+        prev = [v for v in range(len(par)) if par[v] in best and v > max(prev)]
+    for v in range(1, len(par)):
+        lp = _lsm(small[par[v]])[tok[v]]
+        assert abs(edge[v] - lp) < 1e-6
+        path, w = 0.0, v
+        while w:
+            path += _lsm(small[par[w]])[tok[w]]
+            w = par[w]
+        assert abs(score[v] - path) < 1e-5
+
+
+def test_grow_tree_middle_first_step_expands_the_root():
+    rng = synth.make_rng(72)
+    small = synth.normal_f32(rng, (32, 16), 2.0)
+    middle = synth.normal_f32(rng, (32, 16), 2.0)
+    par, tok, edge, score, vis, fr = O.grow_tree([1, 0], 3, 2, small, middle)
+    assert fr[0] == [0] and vis.tolist()[:1] == [1] and vis.sum() == 1
+    top = np.lexsort((np.arange(16), -middle[0].astype(np.float64)))[:2].tolist()
+    assert tok[1:3].tolist() == top and par[1:3].tolist() == [0, 0]
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_grow_tree_random_schedules_invariants(seed):
+    rng = synth.make_rng(73 + seed)
+    V, W, m, D = 24, 3, 2, 5
+    sched = rng.integers(0, 2, size=D).tolist()
+    cap = 1 + D * W * m
+    small = synth.normal_f32(rng, (cap, V), 2.0)
+    middle = synth.normal_f32(rng, (cap, V), 2.0)
+    par, tok, edge, score, vis, fr = O.grow_tree(sched, W, m, small, middle)
+    n = len(par)
+    assert n == 1 + m * sum(len(f) for f in fr)
+    O.check_tree(par)
+    last_mid = max([k for k, a in enumerate(sched) if a == 1], default=-1)
+    # P is every node that existed when the last middle step ran
+    n_then = 1 + m * sum(len(f) for f in fr[:last_mid]) if last_mid >= 0 else 0
+    assert vis.tolist() == [1] * n_then + [0] * (n - n_then)
+    for v in range(1, n):
+        # a visited node carries the middle drafter's edge; an unvisited one
+        # the edge of the drafter whose step created it
+        made_at = next(k for k in range(D) if par[v] in fr[k] and
+                       v < 1 + m * sum(len(f) for f in fr[:k + 1]))
+        table = middle if (vis[v] or sched[made_at] == 1) else small
+        assert abs(edge[v] - _lsm(table[par[v]])[tok[v]]) < 1e-6
+        assert score[v] == np.float32(score[par[v]] + edge[v])
