@@ -63,42 +63,80 @@ __device__ __forceinline__ int scan_pos(int c0, int i, int j, int vw) {
   return c0 + (i * kScanThreads + (int)threadIdx.x) * vw + j;
 }
 
+// One 16-byte vector at an edge of the chunk: elements [pos, pos + VW) that
+// lie below c1 are read one by one, the rest read as -inf.  A rolled loop:
+// only the threads at a chunk edge run it, and it stays small in the
+// instruction cache.
+template <typename T>
+__device__ __forceinline__ uint4 load_edge_vec(const T* __restrict__ row, int pos, int c1) {
+  constexpr int VW = ScanTraits<T>::kVW;
+  constexpr int EB = 16 / VW * 8;  // bits per element
+  uint64_t val[2] = {0ull, 0ull}, got[2] = {0ull, 0ull};
+#pragma unroll 1
+  for (int j = 0; j < VW; ++j) {
+    if (pos + j < c1) {
+      uint64_t x;
+      if constexpr (VW == 8) x = reinterpret_cast<const uint16_t*>(row)[pos + j];
+      else x = reinterpret_cast<const uint32_t*>(row)[pos + j];
+      const int half = j / (VW / 2), sh = EB * (j % (VW / 2));
+      const uint64_t fm = (EB == 64 ? ~0ull : ((1ull << EB) - 1ull)) << sh;
+      if (half) { val[1] |= x << sh; got[1] |= fm; } else { val[0] |= x << sh; got[0] |= fm; }
+    }
+  }
+  const uint64_t neg = (uint64_t)ScanTraits<T>::kNegInfWord * 0x100000001ull;
+  const uint64_t lo = val[0] | (neg & ~got[0]), hi = val[1] | (neg & ~got[1]);
+  return make_uint4((uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)hi, (uint32_t)(hi >> 32));
+}
+
 // Load this thread's elements of [c0, c1); positions past c1 read as -inf.
 // kAligned: the row start is 16-byte aligned (c0 is a multiple of VW).
+// Whole vectors take one 16-byte load each; the few vectors that straddle
+// c1 (or every vector of an unaligned row) are filled afterwards by one
+// rolled fix-up loop, which keeps the unrolled fast path small.
 template <typename T, bool kAligned>
 __device__ __forceinline__ void scan_load(const T* __restrict__ row, int c0, int c1,
                                           uint4 (&buf)[kScanVecs]) {
   constexpr int VW = ScanTraits<T>::kVW;
+  constexpr uint32_t kNeg = ScanTraits<T>::kNegInfWord;
+  uint32_t partial = 0;  // vectors that start below c1 but are not loaded whole
 #pragma unroll
   for (int i = 0; i < kScanVecs; ++i) {
     const int pos = scan_pos(c0, i, 0, VW);
     if (kAligned && pos + VW <= c1) {
       buf[i] = ld_stream_v4(row + pos);
     } else {
-      uint32_t w[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) w[q] = ScanTraits<T>::kNegInfWord;
-      if (pos < c1) {
-        if constexpr (VW == 8) {
-          const uint16_t* r16 = reinterpret_cast<const uint16_t*>(row);
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (pos + j < c1) {
-              const uint32_t h = r16[pos + j];
-              w[j >> 1] = (j & 1) ? ((w[j >> 1] & 0x0000FFFFu) | (h << 16))
-                                  : ((w[j >> 1] & 0xFFFF0000u) | h);
-            }
-          }
-        } else {
-          const uint32_t* r32 = reinterpret_cast<const uint32_t*>(row);
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            if (pos + j < c1) w[j] = r32[pos + j];
-        }
-      }
-      buf[i] = make_uint4(w[0], w[1], w[2], w[3]);
+      buf[i] = make_uint4(kNeg, kNeg, kNeg, kNeg);
+      if (pos < c1) partial |= 1u << i;
     }
   }
+  while (partial) {
+    const int i = __ffs(partial) - 1;
+    partial &= partial - 1;
+    const uint4 v = load_edge_vec<T>(row, scan_pos(c0, i, 0, VW), c1);
+#pragma unroll
+    for (int j = 0; j < kScanVecs; ++j)
+      if (i == j) buf[j] = v;
+  }
+}
+
+// vector i of the thread's buffer for a run-time i (a select chain: keeps
+// the buffer in registers)
+__device__ __forceinline__ uint4 buf_vec(const uint4 (&buf)[kScanVecs], int i) {
+  uint4 q = buf[0];
+#pragma unroll
+  for (int j = 1; j < kScanVecs; ++j)
+    if (i == j) q = buf[j];
+  return q;
+}
+
+// value of element (i, j) of a thread's chunk read back from global memory
+// (rare paths re-read instead of holding code for every register slot)
+template <typename T>
+__device__ __forceinline__ float load_elem(const T* __restrict__ row, int pos) {
+  if constexpr (ScanTraits<T>::kVW == 8)
+    return __uint_as_float((uint32_t)reinterpret_cast<const uint16_t*>(row)[pos] << 16);
+  else
+    return reinterpret_cast<const float*>(row)[pos];
 }
 
 // Largest element of this thread (-inf if it has none).
@@ -196,19 +234,41 @@ __device__ __forceinline__ float scan_thread_sumexp(const uint4 (&buf)[kScanVecs
 }
 
 // Lowest position in [c0, c1) whose value equals v (INT_MAX if none).
+// Positions grow in scan order (vector, then lane), so the first match in
+// that order is the lowest; a match at or past c1 means none below c1.
 template <typename T>
 __device__ __forceinline__ int scan_first_pos(const uint4 (&buf)[kScanVecs], int c0, int c1,
-                                              float v) {
-  constexpr int VW = ScanTraits<T>::kVW;
-  int best = 0x7FFFFFFF;
+                                              float v);
+template <>
+__device__ __forceinline__ int scan_first_pos<float>(const uint4 (&buf)[kScanVecs], int c0, int c1,
+                                                     float v) {
 #pragma unroll
-  for (int i = kScanVecs - 1; i >= 0; --i)
+  for (int i = 0; i < kScanVecs; ++i)
 #pragma unroll
-    for (int j = VW - 1; j >= 0; --j) {
-      const int pos = scan_pos(c0, i, j, VW);
-      if (pos < c1 && vec_elem<T>(buf[i], j) == v) best = pos;
+    for (int j = 0; j < 4; ++j)
+      if (vec_elem<float>(buf[i], j) == v) {
+        const int pos = scan_pos(c0, i, j, 4);
+        return pos < c1 ? pos : 0x7FFFFFFF;
+      }
+  return 0x7FFFFFFF;
+}
+template <>
+__device__ __forceinline__ int scan_first_pos<__nv_bfloat16>(const uint4 (&buf)[kScanVecs], int c0,
+                                                             int c1, float v) {
+  // v is an element value, so it is exact in bf16: one packed compare per pair
+  const __nv_bfloat162 v2 = __float2bfloat162_rn(v);
+#pragma unroll
+  for (int i = 0; i < kScanVecs; ++i)
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const uint32_t x = vec_word(buf[i], w);
+      const uint32_t mk = __heq2_mask(*reinterpret_cast<const __nv_bfloat162*>(&x), v2);
+      if (mk) {
+        const int pos = scan_pos(c0, i, 2 * w, 8) + ((mk & 0xFFFFu) ? 0 : 1);
+        return pos < c1 ? pos : 0x7FFFFFFF;
+      }
     }
-  return best;
+  return 0x7FFFFFFF;
 }
 
 // Combine two (max, sum of 2^(x - max)) pairs.

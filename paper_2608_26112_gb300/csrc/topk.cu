@@ -5,21 +5,33 @@
 // Grid (C, rows) with clusters of C CTAs along x: the C CTAs of a cluster
 // split one row.  Each CTA
 //   1. stages its chunk in registers and takes per-thread (max, sum of
-//      exp(x - max)) - packed bf16x2 max, one exp per element;
-//   2. sorts the 256 thread maxima per warp and picks the value threshold
-//      t = the largest value v with at least k thread maxima >= v.  At
-//      least k elements reach t, and only threads whose max reaches t can
-//      hold elements that do, so candidates are collected by a handful of
-//      threads only;
+//      exp(x - max)) - packed bf16x2 max, one exp per element - merged per
+//      warp with shuffles;
+//   2. sorts the 256 thread maxima per warp; after one barrier each of the
+//      top-k lanes of every warp counts, by binary search in the eight
+//      sorted lists, how many maxima reach its own value, and the largest
+//      value with a count >= k is the threshold t = the k-th largest thread
+//      maximum.  At least k elements reach t, and only threads whose max
+//      reaches t can hold elements that do, so candidates are collected by a
+//      handful of threads only, which visit just the 16-byte vectors whose
+//      packed max reaches t;
 //   3. ranks the candidates by 64-bit keys (value desc, token asc - exact
-//      on ties) into its local top-k.  Heavily tied chunks can overflow the
-//      candidate buffer; they fall back to an exact key threshold (the k-th
-//      largest per-thread (max, first position) key), which bounds the
+//      on ties) by counting larger keys.  Heavily tied chunks can overflow
+//      the candidate buffer; they fall back to an exact key threshold (the
+//      k-th largest per-thread (max, first position) key), which bounds the
 //      candidates by 64 * k;
-//   4. pushes (max, sum, top-k) into the cluster leader's shared memory
-//      (DSMEM stores) and meets the cluster barrier once.
-// The leader merges the C partials into lse and the row's top-k and writes
-// the outputs.  No global scratch and no second launch.
+//   4. the ranking threads store the chunk's top-k (descending) straight
+//      into the cluster leader's shared memory (DSMEM), each warp adds its
+//      (max, sum), and the cluster meets one barrier.
+// In the leader every received key finds its row rank as its index in its
+// own sorted list plus, by binary search, the number of larger keys in each
+// other list; the k keys of rank < k write the outputs, and their warps fold
+// the C * 8 (max, sum) pairs into the lse.  No global scratch and no second
+// launch.
+//
+// These kernels are latency-bound, and several CTAs share an SM: the code
+// keeps dependency chains short and the executed code small (rare paths are
+// rolled loops), so the instruction cache holds the hot path.
 #include <cooperative_groups.h>
 
 #include "launch.h"
@@ -37,18 +49,53 @@ static_assert(kCandMax >= kScanVecs * 8 * kMaxK, "exact fallback must fit the bu
 
 struct TopkSmem {
   uint64_t cand[kCandMax];
-  uint64_t top[kMaxK];
-  uint64_t recv_top[kMaxCluster * kMaxK];  // leader only: partials pushed by the cluster
-  float recv_m[kMaxCluster];
-  float recv_s[kMaxCluster];
-  float warp_v[8 * kMaxK];
+  uint64_t recv_top[kMaxCluster * kMaxK];  // leader only: each CTA's sorted top-k
+  float recv_m[kMaxCluster * 8];           // leader only: each warp's (max, sum)
+  float recv_s[kMaxCluster * 8];
+  float warp_v[8 * 32];  // each warp's 32 thread maxima, sorted descending
   uint64_t warp_k[8 * kMaxK];
-  float red_m[8], red_s[8];
-  uint32_t thr_ord;
   uint64_t thr_key;
+  uint32_t thr_ord;
   int ncand;
-  float lse;
 };
+
+// Entries >= x in the eight descending 32-float lists L[w * 32 ..]: eight
+// branch-free binary searches run in lockstep (5 halving steps and a final
+// probe), so each step issues eight independent shared loads.
+__device__ __forceinline__ int count_ge_8x32(const float* L, float x) {
+  int pos[8];
+#pragma unroll
+  for (int w = 0; w < 8; ++w) pos[w] = 0;
+#pragma unroll
+  for (int step = 16; step > 0; step >>= 1)
+#pragma unroll
+    for (int w = 0; w < 8; ++w) pos[w] += (L[w * 32 + pos[w] + step - 1] >= x) ? step : 0;
+  int cnt = 0;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) cnt += pos[w] + ((L[w * 32 + pos[w]] >= x) ? 1 : 0);
+  return cnt;
+}
+
+// Keys > x in the C descending lists of n <= 32 keys at L[c * n ..], list
+// `skip` excluded: the C binary searches run in lockstep.
+__device__ __forceinline__ int count_gt_lists(const uint64_t* L, int C, int n, int skip,
+                                              uint64_t x) {
+  int pos[kMaxCluster];
+#pragma unroll
+  for (int c = 0; c < kMaxCluster; ++c) pos[c] = 0;
+#pragma unroll
+  for (int step = 16; step > 0; step >>= 1)
+#pragma unroll
+    for (int c = 0; c < kMaxCluster; ++c) {
+      const int i = pos[c] + step - 1;
+      if (c < C && i < n && L[c * n + i] > x) pos[c] += step;
+    }
+  int cnt = 0;
+#pragma unroll
+  for (int c = 0; c < kMaxCluster; ++c)
+    if (c < C && c != skip) cnt += pos[c] + ((pos[c] < n && L[c * n + pos[c]] > x) ? 1 : 0);
+  return cnt;
+}
 
 // descending bitonic sort of one value per lane; lane j ends with the j-th largest
 template <typename K>
@@ -66,6 +113,116 @@ __device__ __forceinline__ K warp_sort_desc(K x) {
   return x;
 }
 
+__device__ __forceinline__ void push_cand(TopkSmem& sm, uint64_t key) {
+  const int slot = atomicAdd(&sm.ncand, 1);
+  if (slot < kCandMax) sm.cand[slot] = key;
+}
+
+// Elements >= tv of this thread's chunk into the candidate buffer.  Only the
+// vectors whose packed max reaches tv are visited (typically one).
+template <typename T>
+__device__ __forceinline__ void collect_candidates(const uint4 (&buf)[kScanVecs], int c0, int c1,
+                                                   float tv, TopkSmem& sm) {
+  constexpr int VW = ScanTraits<T>::kVW;
+  uint32_t hit = 0;
+  if constexpr (VW == 8) {
+    // tv is a thread max, so it is exactly representable in bf16
+    const __nv_bfloat162 tv2 = __float2bfloat162_rn(tv);
+#pragma unroll
+    for (int i = 0; i < kScanVecs; ++i) {
+      const uint4 q = buf[i];
+      const __nv_bfloat162 m2 =
+          __hmax2(__hmax2(*reinterpret_cast<const __nv_bfloat162*>(&q.x),
+                          *reinterpret_cast<const __nv_bfloat162*>(&q.y)),
+                  __hmax2(*reinterpret_cast<const __nv_bfloat162*>(&q.z),
+                          *reinterpret_cast<const __nv_bfloat162*>(&q.w)));
+      hit |= (__hge2_mask(m2, tv2) ? 1u : 0u) << i;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < kScanVecs; ++i) {
+      const uint4 q = buf[i];
+      const float m = fmaxf(fmaxf(__uint_as_float(q.x), __uint_as_float(q.y)),
+                            fmaxf(__uint_as_float(q.z), __uint_as_float(q.w)));
+      hit |= (m >= tv ? 1u : 0u) << i;
+    }
+  }
+  while (hit) {
+    const int i = __ffs(hit) - 1;
+    hit &= hit - 1;
+    const uint4 q = buf_vec(buf, i);
+    // bit j: element j of the vector reaches tv (independent compares)
+    uint32_t em = 0;
+    if constexpr (VW == 8) {
+      const __nv_bfloat162 tv2 = __float2bfloat162_rn(tv);
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const uint32_t x = vec_word(q, w);
+        const uint32_t mk = __hge2_mask(*reinterpret_cast<const __nv_bfloat162*>(&x), tv2);
+        em |= ((mk & 1u) | ((mk >> 15) & 2u)) << (2 * w);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) em |= (__uint_as_float(vec_word(q, j)) >= tv ? 1u : 0u) << j;
+    }
+    while (em) {
+      const int j = __ffs(em) - 1;
+      em &= em - 1;
+      const uint32_t w = vec_word(q, VW == 8 ? (j >> 1) : j);
+      const float v = VW == 8 ? ((j & 1) ? bf16_hi(w) : bf16_lo(w)) : __uint_as_float(w);
+      const int pos = scan_pos(c0, i, j, VW);
+      if (pos < c1) push_cand(sm, make_key(v, (uint32_t)pos));
+    }
+  }
+}
+
+// Heavy ties (the candidate buffer overflowed): exact key threshold = the
+// k-th largest per-thread (max, first position) key; candidates are the
+// elements whose key reaches it (at most 64 * k).  The chunk is re-read from
+// global memory in rolled loops: this path is rare and stays out of the hot
+// code.  Called by every thread of the CTA; returns the candidate count.
+template <typename T>
+__device__ __noinline__ int tie_fallback(const T* __restrict__ rowp, int c0, int c1, int k,
+                                         float tmax, TopkSmem& sm) {
+  constexpr int VW = ScanTraits<T>::kVW;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  __syncthreads();  // every thread has read ncand before it is reset below
+  int fp = 0x7FFFFFFF;
+#pragma unroll 1
+  for (int e = 0; e < kScanVecs * VW && fp == 0x7FFFFFFF; ++e) {
+    const int pos = scan_pos(c0, e / VW, e % VW, VW);
+    if (pos < c1 && load_elem<T>(rowp, pos) == tmax) fp = pos;
+  }
+  const uint64_t tk = (fp == 0x7FFFFFFF) ? 0ull : make_key(tmax, (uint32_t)fp);
+  const uint64_t sk = warp_sort_desc<uint64_t>(tk);
+  if (lane < k) sm.warp_k[warp * k + lane] = sk;
+  if (tid == 0) {
+    sm.thr_key = 0ull;
+    sm.ncand = 0;
+  }
+  __syncthreads();
+  if (tid < 8 * k) {
+    const uint64_t mine = sm.warp_k[tid];
+    int rank = 0;
+    for (int i = 0; i < 8 * k; ++i) rank += (sm.warp_k[i] > mine) ? 1 : 0;
+    if (mine != 0ull && rank == k - 1) sm.thr_key = mine;
+  }
+  __syncthreads();
+  const uint64_t thr = sm.thr_key;
+  if (tk >= thr && tk != 0ull) {
+#pragma unroll 1
+    for (int e = 0; e < kScanVecs * VW; ++e) {
+      const int pos = scan_pos(c0, e / VW, e % VW, VW);
+      if (pos < c1) {
+        const uint64_t key = make_key(load_elem<T>(rowp, pos), (uint32_t)pos);
+        if (key >= thr) push_cand(sm, key);
+      }
+    }
+  }
+  __syncthreads();
+  return min(sm.ncand, kCandMax);
+}
+
 template <typename T, bool kAligned>
 __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a) {
   __shared__ TopkSmem sm;
@@ -77,6 +234,7 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   const int k = a.k;
   const int V = a.V;
   constexpr int VW = ScanTraits<T>::kVW;
+  const float NEG_INF = __int_as_float(0xff800000);
 
   pdl_launch_dependents();
   pdl_wait();
@@ -88,10 +246,10 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
     return;
   }
   cluster_arrive_relaxed();
-  // the leader's output threads fetch the parent's path score now, while
-  // the logits are in flight
+  // the leader's threads fetch the parent's path score now, while the
+  // logits are in flight (one broadcast request per warp)
   float parent_score = 0.f;
-  if (crank == 0 && tid < k) parent_score = __ldg(a.parent_score + row);
+  if (crank == 0) parent_score = __ldg(a.parent_score + row);
   const int per = ((V + C - 1) / C + VW - 1) / VW * VW;
   const int c0 = min(V, crank * per);
   const int c1 = min(V, c0 + per);
@@ -100,10 +258,9 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   uint4 buf[kScanVecs];
   scan_load<T, kAligned>(rowp, c0, c1, buf);
   if (tid == 0) {
-    sm.thr_ord = 0u;
     sm.ncand = 0;
+    sm.thr_ord = 0u;
   }
-  if (tid < kMaxK) sm.top[tid] = 0ull;
 
   // 1. per-thread max and exp-sum, warp-combined
   const float tmax = scan_thread_max<T>(buf);
@@ -114,149 +271,69 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
     const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
     lse_merge(m, s, m2, s2);
   }
-  // 2. value threshold from the sorted thread maxima
+  // 2. value threshold: the k-th largest of the 256 thread maxima.  It is
+  //    among the top k of some warp's sorted list; each such entry counts
+  //    the maxima >= itself in all eight lists, and the largest entry with
+  //    a count >= k is the k-th largest.
   const float sv = warp_sort_desc<float>(tmax);
-  if (lane < k) sm.warp_v[warp * k + lane] = sv;
-  if (lane == 0) {
-    sm.red_m[warp] = m;
-    sm.red_s[warp] = s;
-  }
+  sm.warp_v[warp * 32 + lane] = sv;
   __syncthreads();
-  if (tid < 8 * k) {
-    const float v = sm.warp_v[tid];
-    int ge = 0;
-    for (int i = 0; i < 8 * k; ++i) ge += (sm.warp_v[i] >= v) ? 1 : 0;
-    if (ge >= k && v == v) atomicMax(&sm.thr_ord, ord_f32(v));
-  }
+  if (lane < k && count_ge_8x32(sm.warp_v, sv) >= k) atomicMax(&sm.thr_ord, ord_f32(sv));
   __syncthreads();
   const float tv = unord_f32(sm.thr_ord);
   // 3. candidates (only threads whose max reaches the threshold have any)
-  if (tmax >= tv) {
-    auto push = [&](float v, int pos) {
-      if (pos < c1) {
-        const int slot = atomicAdd(&sm.ncand, 1);
-        if (slot < kCandMax) sm.cand[slot] = make_key(v, (uint32_t)pos);
-      }
-    };
-    if constexpr (VW == 8) {
-      // one packed compare per element pair; tv is a thread max, so it is
-      // exactly representable in bf16
-      const __nv_bfloat162 tv2 = __float2bfloat162_rn(tv);
-#pragma unroll
-      for (int i = 0; i < kScanVecs; ++i)
-#pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          const uint32_t x = vec_word(buf[i], w);
-          const uint32_t mk = __hge2_mask(*reinterpret_cast<const __nv_bfloat162*>(&x), tv2);
-          if (mk) {
-            const int pos = scan_pos(c0, i, 2 * w, VW);
-            if (mk & 0xFFFFu) push(bf16_lo(x), pos);
-            if (mk >> 16) push(bf16_hi(x), pos + 1);
-          }
-        }
-    } else {
-#pragma unroll
-      for (int i = 0; i < kScanVecs; ++i)
-#pragma unroll
-        for (int j = 0; j < VW; ++j) {
-          const float v = vec_elem<T>(buf[i], j);
-          if (v >= tv) push(v, scan_pos(c0, i, j, VW));
-        }
-    }
-  }
+  if (tmax >= tv) collect_candidates<T>(buf, c0, c1, tv, sm);
   __syncthreads();
   int nc = sm.ncand;
-  if (nc > kCandMax) {
-    // heavy ties: exact key threshold = k-th largest (thread max, first position)
-    __syncthreads();  // every thread has read ncand before it is reset below
-    const int fp = (c0 + (int)tid * VW >= c1) ? 0x7FFFFFFF : scan_first_pos<T>(buf, c0, c1, tmax);
-    const uint64_t tk = (fp == 0x7FFFFFFF) ? 0ull : make_key(tmax, (uint32_t)fp);
-    const uint64_t sk = warp_sort_desc<uint64_t>(tk);
-    if (lane < k) sm.warp_k[warp * k + lane] = sk;
-    if (tid == 0) {
-      sm.thr_key = 0ull;
-      sm.ncand = 0;
-    }
-    __syncthreads();
-    if (tid < 8 * k) {
-      const uint64_t mine = sm.warp_k[tid];
-      int rank = 0;
-      for (int i = 0; i < 8 * k; ++i) rank += (sm.warp_k[i] > mine) ? 1 : 0;
-      if (mine != 0ull && rank == k - 1) sm.thr_key = mine;
-    }
-    __syncthreads();
-    const uint64_t thr = sm.thr_key;
-    if (tk >= thr && tk != 0ull) {
-#pragma unroll
-      for (int i = 0; i < kScanVecs; ++i)
-#pragma unroll
-        for (int j = 0; j < VW; ++j) {
-          const int pos = scan_pos(c0, i, j, VW);
-          const uint64_t key = make_key(vec_elem<T>(buf[i], j), (uint32_t)pos);
-          if (pos < c1 && key >= thr) {
-            const int slot = atomicAdd(&sm.ncand, 1);
-            if (slot < kCandMax) sm.cand[slot] = key;
-          }
-        }
-    }
-    __syncthreads();
-    nc = min(sm.ncand, kCandMax);
-  }
+  if (nc > kCandMax) nc = tie_fallback<T>(rowp, c0, c1, k, tmax, sm);
+
+  // 4. rank the candidates and store the chunk's top-k (descending) straight
+  //    into the leader's receive slots; slots past the candidates get 0
+  cluster_wait();  // every CTA of the cluster is running: DSMEM is addressable
+  TopkSmem* lead = cluster.map_shared_rank(&sm, 0);
+  uint64_t* dst = lead->recv_top + crank * k;
   for (int i = tid; i < nc; i += kScanThreads) {
     const uint64_t mine = sm.cand[i];
     int rank = 0;
+#pragma unroll 4
     for (int j = 0; j < nc; ++j) rank += (sm.cand[j] > mine) ? 1 : 0;
-    if (rank < k) sm.top[rank] = mine;
+    if (rank < k) dst[rank] = mine;
   }
-  __syncthreads();
-
-  // 4. push the partial into the leader's shared memory
-  cluster_wait();
-  TopkSmem* lead = cluster.map_shared_rank(&sm, 0);
-  if (tid < k) lead->recv_top[crank * k + tid] = sm.top[tid];
-  if (tid == 0) {
-    float M = sm.red_m[0], S = sm.red_s[0];
-#pragma unroll
-    for (int w = 1; w < 8; ++w) lse_merge(M, S, sm.red_m[w], sm.red_s[w]);
-    lead->recv_m[crank] = M;
-    lead->recv_s[crank] = S;
+  if (tid >= nc && tid < k) dst[tid] = 0ull;
+  if (lane == 0) {
+    lead->recv_m[crank * 8 + warp] = m;
+    lead->recv_s[crank * 8 + warp] = s;
   }
   cluster.sync();
   if (crank != 0) return;
 
-  // ---- leader: merge the C partials
-  if (warp == 0) {
-    // lse over the C partials: one (max, sum) per lane, shuffle tree
-    float M = lane < C ? sm.recv_m[lane] : __int_as_float(0xff800000);
-    float S = lane < C ? sm.recv_s[lane] : 0.f;
+  // ---- leader: key t (list c = t / k, index j = t % k) has row rank
+  // j + the number of larger keys in the other lists (keys are unique; empty
+  // slots are 0 and never reach rank k, as the row has >= k real keys)
+  const int ck = C * k;
+  if (warp * 32 >= ck) return;
+  float M = NEG_INF, S = 0.f;
+  for (int i = lane; i < C * 8; i += 32) lse_merge(M, S, sm.recv_m[i], sm.recv_s[i]);
 #pragma unroll
-    for (int o = 8; o > 0; o >>= 1) {
-      const float m2 = __shfl_xor_sync(0xffffffffu, M, o);
-      const float s2 = __shfl_xor_sync(0xffffffffu, S, o);
-      lse_merge(M, S, m2, s2);
-    }
-    if (lane == 0) {
-      const float lse = (M == __int_as_float(0xff800000)) ? M : M + log2f(S) * kLn2;
-      sm.lse = lse;
-      if (a.lse_out) a.lse_out[row] = lse;
-    }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, M, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, S, o);
+    lse_merge(M, S, m2, s2);
   }
-  for (int t = tid; t < C * k; t += kScanThreads) {
-    const uint64_t mine = sm.recv_top[t];
-    int rank = 0;
-    for (int j = 0; j < C * k; ++j) rank += (sm.recv_top[j] > mine) ? 1 : 0;
-    if (rank < k) sm.top[rank] = mine;
-  }
-  __syncthreads();
-  if (tid < k) {
-    const uint64_t key = sm.top[tid];
-    const float v = key_value(key);
-    const float lse = sm.lse;
-    const float lp = (lse == __int_as_float(0xff800000)) ? lse : (v - lse);
-    const size_t o = (size_t)row * k + tid;
-    a.tok[o] = (int32_t)key_index(key);
-    a.logprob[o] = lp;
-    a.score[o] = __fadd_rn(parent_score, lp);
+  const float lse = (M == NEG_INF) ? M : M + log2f(S) * kLn2;
+  for (int t = tid; t < ck; t += kScanThreads) {
+    const uint64_t key = sm.recv_top[t];
+    const int c = t / k;
+    const int rank = t - c * k + count_gt_lists(sm.recv_top, C, k, c, key);
+    if (key != 0ull && rank < k) {
+      const float v = key_value(key);
+      const float lp = (lse == NEG_INF) ? lse : (v - lse);
+      const size_t o = (size_t)row * k + rank;
+      a.tok[o] = (int32_t)key_index(key);
+      a.logprob[o] = lp;
+      a.score[o] = __fadd_rn(parent_score, lp);
+      if (rank == 0 && a.lse_out) a.lse_out[row] = lse;
+    }
   }
 }
 
