@@ -249,9 +249,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t p_base = smem_u32(smem + L::kOffP);
   const float NEG_INF = __int_as_float(0xff800000);
 
-  // the next kernel on the stream may be dispatched now (it waits for this
-  // grid's completion before touching memory)
+  // the next kernel on the stream may be dispatched now; this one's global
+  // reads wait for the previous kernel (a no-op without programmatic
+  // dependent launch)
   pdl_launch_dependents();
+  pdl_wait();
   // ---- the tree's extent (global reads in flight while the barriers are set up)
   const int off = a.node_off[b];
   const int n = a.node_off[b + 1] - off;
@@ -700,7 +702,9 @@ cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtenso
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = L::kAlloc;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  // programmatic dependent launch: this launch is dispatched while the
+  // previous kernel on the stream finishes (its reads wait in the kernel)
+  cudaLaunchAttribute attr[2];
   if (plan.coop) {
     attr[0].id = cudaLaunchAttributeCooperative;
     attr[0].val.cooperative = 1;
@@ -710,8 +714,10 @@ cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtenso
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
   }
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, tq, tk, tv, a);
 }
 
