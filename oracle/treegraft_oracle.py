@@ -12,7 +12,8 @@ Every function is pinned against something other than itself by the
 CPU-only tests in tests/test_oracle_pins.py (brute force, closed forms,
 invariants).  Parity status per function:
   ancestor_mask, tree_attention, expand_topk, rescore_select, accept,
-  global_prune, grow_tree: pinned.
+  global_prune, grow_state / grow_step / grow_tree: pinned (grow_tree is
+  grow_step applied over a schedule; its pins exercise every branch of it).
 
 Readings of the paper taken here (where it is silent or loose):
   * depth(root) = 0; mask row u has P + depth(u) + 1 ones (Algorithm 3 mask:
@@ -340,65 +341,80 @@ def _row_log_softmax(logits, r: int, bf16: bool):
     return x, lse
 
 
-def grow_tree(schedule, W: int, m: int, small_logits, middle_logits, *, bf16: bool = False):
-    """TreeGraft shared-tree construction (Algorithm 2) for one sequence.
+def grow_state():
+    """Initial shared tree of Algorithm 2: the root alone, N_1 = {r}, P_1 empty,
+    s(r) = 0 (log of 1)."""
+    return dict(parent=[-1], token=[0], edge=[np.float32(0.0)], score=[np.float32(0.0)],
+                new=[0], P=set(), lse_m={})
+
+
+def grow_step(state, a: int, W: int, m: int, small_logits, middle_logits, *, bf16: bool = False):
+    """One drafting step k of Algorithm 2 on `state` (see grow_state), in place.
 
     The drafters' next-token logits under the prefix ending at node v are
     rows v of small_logits and middle_logits (tables indexed by node id, the
-    stand-in for the drafter forwards).  Scores are log-domain: s(root) = 0,
-    s(u) = fp32(s(v) + p(u)) with p(u) = fp32(l_u - lse) the drafter's
-    log-probability of u's token.  Step k with schedule[k] = 0 (small
-    drafter): C = N_k (the nodes made at the previous step; {root} at
-    first), F = Top_W(C, s) by (s desc, id asc), and each v in F gets its
-    m best small-drafter tokens (logit desc, token asc) as new children.
-    schedule[k] = 1 (middle drafter): C = V(T) \\ P; every non-root v in C is
-    rescored, p(v) = fp32(l_m[pa(v), token(v)] - lse_m[pa(v)]), and s is
-    recomputed in node order; F = Top_W(C, s); each v in F gets its m best
-    middle-drafter tokens; then P = P u C.  Children are appended in frontier
-    order, then child rank, never replacing an existing node.
+    stand-in for the drafter forwards).  Scores are log-domain: s(u) =
+    fp32(s(v) + p(u)) with p(u) = fp32(l_u - lse) the drafter's
+    log-probability of u's token.  a = 0 (small drafter): C = N_k (the nodes
+    made at the previous step), F = Top_W(C, s) by (s desc, id asc), and
+    each v in F gets its m best small-drafter tokens (logit desc, token asc)
+    as new children.  a = 1 (middle drafter): C = V(T) \\ P; the log-sum-exp
+    of every row in C is taken (and cached: it is the forward pass over C);
+    every non-root v in C is rescored, p(v) = fp32(l_m[pa(v), token(v)] -
+    lse_m[pa(v)]), and s is recomputed in node order; F = Top_W(C, s); each
+    v in F gets its m best middle-drafter tokens; then P = P u C.  Children
+    are appended in frontier order, then child rank, never replacing an
+    existing node.  Returns the frontier F.
+    """
+    parent, token, edge, score = state["parent"], state["token"], state["edge"], state["score"]
+    P, lse_m = state["P"], state["lse_m"]
+    n = len(parent)
+    if a == 0:
+        C = list(state["new"])
+        table = small_logits
+    else:
+        C = [v for v in range(n) if v not in P]
+        for v in C:
+            lse_m[v] = _row_log_softmax(middle_logits, v, bf16)[1]
+        for v in C:
+            if v == 0:
+                continue
+            row = _row_values(middle_logits, parent[v], bf16)
+            edge[v] = np.float32(row[token[v]] - lse_m[parent[v]])
+            score[v] = np.float32(score[parent[v]] + edge[v])
+        table = middle_logits
+    F = sorted(C, key=lambda v: (-float(score[v]), v))[:W]
+    made = []
+    for v in F:
+        x, lse = _row_log_softmax(table, v, bf16)
+        order = np.lexsort((np.arange(len(x)), -x))[:m]
+        for y in order:
+            lp = np.float32(x[y] - lse)
+            parent.append(v)
+            token.append(int(y))
+            edge.append(lp)
+            score.append(np.float32(score[v] + lp))
+            made.append(len(parent) - 1)
+    if a == 1:
+        P.update(C)
+    state["new"] = made
+    return F
+
+
+def grow_tree(schedule, W: int, m: int, small_logits, middle_logits, *, bf16: bool = False):
+    """TreeGraft shared-tree construction (Algorithm 2) for one sequence: the
+    steps of `schedule` (0 = small drafter, 1 = middle drafter) applied in
+    order by grow_step from the root alone.
 
     Returns parent int32, token int32, edge f32, score f32 (per node), the
     visited set P as uint8, and the list of frontiers (one per step).
     """
-    parent, token = [-1], [0]
-    edge, score = [np.float32(0.0)], [np.float32(0.0)]
-    new = [0]
-    P = set()
-    lse_m = {}
-    frontiers = []
-    for a in schedule:
-        n = len(parent)
-        if a == 0:
-            C = list(new)
-            table = small_logits
-        else:
-            C = [v for v in range(n) if v not in P]
-            for v in C:
-                lse_m[v] = _row_log_softmax(middle_logits, v, bf16)[1]
-            for v in C:
-                if v == 0:
-                    continue
-                row = _row_values(middle_logits, parent[v], bf16)
-                edge[v] = np.float32(row[token[v]] - lse_m[parent[v]])
-                score[v] = np.float32(score[parent[v]] + edge[v])
-            table = middle_logits
-        F = sorted(C, key=lambda v: (-float(score[v]), v))[:W]
-        frontiers.append(F)
-        made = []
-        for v in F:
-            x, lse = _row_log_softmax(table, v, bf16)
-            order = np.lexsort((np.arange(len(x)), -x))[:m]
-            for y in order:
-                lp = np.float32(x[y] - lse)
-                parent.append(v)
-                token.append(int(y))
-                edge.append(lp)
-                score.append(np.float32(score[v] + lp))
-                made.append(len(parent) - 1)
-        if a == 1:
-            P.update(C)
-        new = made
+    state = grow_state()
+    frontiers = [grow_step(state, a, W, m, small_logits, middle_logits, bf16=bf16)
+                 for a in schedule]
+    parent = state["parent"]
     visited = np.zeros(len(parent), dtype=np.uint8)
-    visited[sorted(P)] = 1
-    return (np.asarray(parent, np.int32), np.asarray(token, np.int32),
-            np.asarray(edge, np.float32), np.asarray(score, np.float32), visited, frontiers)
+    visited[sorted(state["P"])] = 1
+    return (np.asarray(parent, np.int32), np.asarray(state["token"], np.int32),
+            np.asarray(state["edge"], np.float32), np.asarray(state["score"], np.float32),
+            visited, frontiers)
