@@ -216,6 +216,68 @@ def prune_timing(R, seed, dev, stream, reps):
             "in_step": False, "note": "Algorithm 3 on the pre-pruning tree, latency-bound"}
 
 
+GROW_SCHEDULE = [1, 0, 1, 0, 1]
+
+
+def grow_timing(seed, dev, stream, reps, n_sets=3):
+    """The shared-tree construction (Algorithm 2) timed beside the step, not
+    inside it: the fixed schedule [1, 0, 1, 0, 1] of the paper's ablation
+    (middle, small, middle, small, middle drafter) with frontier W = 10 and
+    branching m = 10, on seeded N(0, 3^2) bf16 drafter tables over the
+    Llama-3 vocabulary (128256); one tree, grown from its root to 411
+    nodes.  Each loop is 5 grow_step calls (15 launches); n_sets table pairs
+    rotate so the 85 MB of rows a loop scans come from HBM."""
+    import numpy as np
+    import torch
+    import paper_2608_26112_gb300 as tg
+    from paper_2608_26112_gb300 import synth
+
+    W = m = 10
+    V = 128256
+    sizes, n, new_lo, n_vis = [], 1, 0, 0
+    for a in GROW_SCHEDULE:
+        pool_lo = new_lo if a == 0 else n_vis
+        sizes.append((a, n, pool_lo))
+        if a == 1:
+            n_vis = n
+        new_lo, n = n, n + min(W, n - pool_lo) * m
+    cap = n
+    rows = sum((1 if a == 0 else 0) * min(W, n_ - lo) + (1 if a == 1 else 0) * (n_ - lo)
+               for a, n_, lo in sizes)
+    sets = []
+    for r in range(n_sets):
+        rng = synth.make_rng(30_000 + seed + r)
+        tabs = [torch.from_numpy(synth.f32_to_bf16_bits(synth.normal_f32(rng, (cap, V), 3.0))
+                                 .view(np.int16)).to(dev).view(torch.bfloat16) for _ in range(2)]
+        tree = dict(parent=torch.full((1, cap), -1, dtype=torch.int32, device=dev),
+                    token=torch.zeros(1, cap, dtype=torch.int32, device=dev),
+                    edge=torch.zeros(1, cap, dtype=torch.float32, device=dev),
+                    score=torch.zeros(1, cap, dtype=torch.float32, device=dev),
+                    lse=torch.zeros(1, cap, dtype=torch.float32, device=dev),
+                    fr=torch.empty(1, W, dtype=torch.int32, device=dev),
+                    ws=tg.grow_workspace(1, cap, m, dev))
+        sets.append((tabs, tree))
+
+    def loop(tabs, t):
+        for a, n_, lo in sizes:
+            tg.grow_step(a, tabs[a], W, m, t["parent"], t["token"], t["edge"], t["score"], n_, lo,
+                         lse_mid=t["lse"], frontier=t["fr"], ws=t["ws"], stream=stream)
+
+    with torch.cuda.stream(stream):
+        for tabs, t in sets:
+            loop(tabs, t)
+    stream.synchronize()
+    g = capture(lambda: [loop(tabs, t) for tabs, t in sets], stream)
+    g.replay()
+    loops = max(5, reps // 10)
+    t = time_graph(g, loops, stream) / (loops * n_sets)
+    b = rows * V * 2
+    return {"us": t * 1e6, "schedule": GROW_SCHEDULE, "W": W, "m": m, "vocab": V,
+            "nodes_out": cap, "rows_scanned": rows, "bytes": b, "GBps": b / t / 1e9,
+            "launches": 3 * len(GROW_SCHEDULE), "in_step": False,
+            "note": "Algorithm 2 grow loop; bytes = drafter-table rows scanned x V x 2"}
+
+
 # --------------------------------------------------------------------------- clocks
 
 class ClockSampler:
@@ -483,6 +545,7 @@ def ours_arm(args):
             g.replay()
             kt[name] = time_graph(g, kreps, stream) / (kreps * R)
         prune = prune_timing(R, rank_seed(args.seed, rank), dev, stream, kreps)
+        grow = grow_timing(rank_seed(args.seed, rank), dev, stream, kreps)
     assert tg.last_device_status(stream) == 0
     t_max = max_over_ranks(t_steps, world)
     steps_per_s = job_throughput(world, K, t_max)
@@ -498,6 +561,7 @@ def ours_arm(args):
         if f:
             kernels[name]["TFLOPs"] = f / kt[name] / 1e12
     kernels["global_prune"] = prune
+    kernels["grow_loop"] = grow
     dom = max(KERNELS, key=lambda n: kt[n])
     b, f = costs[dom]
     achieved = b / kt[dom] / 1e9

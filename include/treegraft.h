@@ -279,6 +279,65 @@ int treegraft_global_prune(const float* score, const int32_t* parent, const int3
                            void* stream);
 
 /*
+ * treegraft_grow_step - one drafting step of the shared draft tree.
+ *
+ * Paper: Algorithm 2 (TreeGraft shared-tree construction with grafting), one
+ * iteration k; with small-drafter steps only it is Algorithm 1.  Scores are
+ * log-probabilities (s(root) = 0, s(u) = fp32(s(v) + p(u)), p(u) the
+ * drafter's natural-log probability of u's token after the prefix ending at
+ * v); Top_W ranks nodes by (s desc, id asc), Top_m tokens by (logit desc,
+ * token asc).
+ *   mode 0 (small drafter): candidate pool C = N_k, the nodes the previous
+ *     step made; F = Top_W(C, s); every v in F gets the m best tokens of its
+ *     row of `logits` (the small drafter's table) as children.
+ *   mode 1 (middle drafter): C = V(T) \ P; the row of every v in C is
+ *     log-softmax normalised and its log-sum-exp cached in lse_mid[v]; every
+ *     non-root v in C is rescored, p(v) = l[pa(v), token(v)] - lse_mid[pa(v)]
+ *     (its parent's middle-drafter row, visited or not), and s is recomputed
+ *     root-first; F = Top_W(C, s); every v in F gets the m best tokens of its
+ *     row.  Then P = P u C.
+ * Children are appended after the last node, in frontier order then child
+ * rank, without replacing any node (a duplicate token is a new sibling).
+ *
+ * Trees: B trees of capacity `cap` (1 <= cap <= TG_MAX_GROW_NODES); tree b
+ * owns rows [b * cap, (b + 1) * cap) of parent, token, edge, score, lse_mid
+ * and of the logit table, with local ids.  All trees grow in lock step with
+ * one schedule, so the sizes are the caller's (host) numbers:
+ *   n        nodes per tree before the step (>= 1: the root alone is n = 1,
+ *            parent[0] = -1, score[0] = 0, edge[0] = 0);
+ *   pool_lo  the pool is [pool_lo, n).  mode 0: the first node the previous
+ *            step made (0 at the first step, where N_1 = {root}).  mode 1:
+ *            |P|, the node count when the last middle step ran (0 if none) -
+ *            P is always the prefix [0, |P|) of the ids, because a middle
+ *            step visits every node that exists and nodes are only appended.
+ * After the step each tree has n + min(W, n - pool_lo) * m nodes (must be
+ * <= cap), the next small step pools [n, that), and after a middle step
+ * |P| = n.
+ * logits   [B * cap, ld] bf16 or fp32: row b * cap + v is the drafter's
+ *          next-token logits after node v of tree b (its forward over the
+ *          tree); V <= ld columns used.
+ * parent, token int32, edge, score fp32 [B * cap]: the tree, updated in place
+ *          (the pool's edge and score are rewritten by a middle step).
+ * lse_mid  fp32 [B * cap]: log-sum-exp of the middle drafter's rows, written
+ *          for the pool by a middle step and read for visited parents; may
+ *          be NULL if mode is 0.
+ * frontier int32 [B, W]: F in rank order, -1 padded.
+ * ws       scratch of treegraft_grow_workspace_size(B, cap, m) bytes,
+ *          16-byte aligned; no initial contents required.
+ * Errors: TG_ERR_INVALID_ARG (null pointer, sizes, capacity overflow),
+ * TG_ERR_UNSUPPORTED (cap > TG_MAX_GROW_NODES, m > TG_MAX_TOPK, vocabulary
+ * above 262144 bf16 / 131072 fp32), TG_ERR_CUDA.  A malformed parent array
+ * sets TG_ERR_DEVICE_TREE, a token outside [0, V) in a middle pool sets
+ * TG_ERR_DEVICE_INDEX; the step's outputs are then undefined.
+ */
+#define TG_MAX_GROW_NODES 1024
+size_t treegraft_grow_workspace_size(int B, int cap, int m);
+int treegraft_grow_step(int mode, const void* logits, int dtype, int V, int64_t ld, int B, int cap,
+                        int n, int pool_lo, int W, int m, int32_t* parent, int32_t* token,
+                        float* edge, float* score, float* lse_mid, int32_t* frontier, void* ws,
+                        size_t ws_bytes, void* stream);
+
+/*
  * treegraft_last_device_status - synchronise `stream`, return the OR of the
  * device status bits raised since the last call on the current device
  * (TG_OK if none), and clear them.  Returns TG_ERR_CUDA if the

@@ -21,6 +21,7 @@ TG_BF16, TG_F32 = 0, 1
 MAX_TREE_NODES = 256
 MAX_TOPK = 32
 MAX_PRUNE_NODES = 1024
+MAX_GROW_NODES = 1024
 
 _lib = None
 
@@ -52,10 +53,15 @@ _SIGNATURES = {
                                  _c_int, _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp],
     "treegraft_global_prune": [_c_vp, _c_vp, _c_vp, _c_int, _c_int, _c_int, _c_int, _c_int,
                                _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp],
+    "treegraft_grow_workspace_size": [_c_int, _c_int, _c_int],
+    "treegraft_grow_step": [_c_int, _c_vp, _c_int, _c_int, _c_i64, _c_int, _c_int, _c_int, _c_int,
+                            _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp,
+                            _c_size, _c_vp],
     "treegraft_last_device_status": [_c_vp],
     "treegraft_status_string": [_c_int],
 }
 _RESTYPES = {"treegraft_accept_workspace_size": _c_size,
+             "treegraft_grow_workspace_size": _c_size,
              "treegraft_tree_attn_workspace_size": _c_size,
              "treegraft_status_string": ctypes.c_char_p}
 
@@ -299,3 +305,47 @@ def global_prune(score, parent, node_off, max_nodes, budget, path_cap, *, out=No
                                       _ptr(paths), _ptr(n_paths), _stream(stream))
     _check("treegraft_global_prune", st)
     return kept, n_kept, new_parent, position, mask, paths, n_paths
+
+
+def grow_workspace(B, cap, m, device):
+    """Scratch for grow_step on B trees of capacity cap with m children per
+    frontier node (uint8 tensor)."""
+    nbytes = int(lib().treegraft_grow_workspace_size(int(B), int(cap), int(m)))
+    if nbytes == 0:
+        raise ValueError("grow workspace: unsupported sizes")
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+def grow_step(mode, logits, W, m, parent, token, edge, score, n, pool_lo, *, lse_mid=None,
+              frontier=None, ws=None, V=None, stream=None):
+    """One drafting step of the shared tree (Algorithm 2; mode 0 = small
+    drafter, 1 = middle drafter) on B trees of capacity cap: parent / token
+    int32 and edge / score fp32 [B, cap] (updated in place), lse_mid fp32
+    [B, cap], logits [B * cap, ld] bf16/fp32 (row b * cap + v follows node v
+    of tree b).  n and pool_lo are the host-side sizes of the step (see
+    treegraft_grow_step).  Returns the frontier int32 [B, W]."""
+    for t, nm in ((parent, "parent"), (token, "token")):
+        _need(t, torch.int32, nm)
+    for t, nm in ((edge, "edge"), (score, "score")):
+        _need(t, torch.float32, nm)
+    if lse_mid is not None:
+        _need(lse_mid, torch.float32, "lse_mid")
+    if parent.dim() != 2:
+        raise ValueError("tree arrays must be [B, cap]")
+    B, cap = parent.shape
+    if logits.dim() != 2 or logits.stride(1) != 1 or not logits.is_cuda:
+        raise ValueError("logits must be a 2-D CUDA tensor with unit column stride")
+    dt = _logit_dtype(logits)
+    V = logits.shape[1] if V is None else int(V)
+    dev = parent.device
+    if frontier is None:
+        frontier = torch.empty(B, int(W), dtype=torch.int32, device=dev)
+    _need(frontier, torch.int32, "frontier")
+    if ws is None:
+        ws = grow_workspace(B, cap, m, dev)
+    st = lib().treegraft_grow_step(int(mode), _ptr(logits), dt, V, logits.stride(0), B, cap, int(n),
+                                   int(pool_lo), int(W), int(m), _ptr(parent), _ptr(token),
+                                   _ptr(edge), _ptr(score), _ptr(lse_mid), _ptr(frontier), _ptr(ws),
+                                   ws.numel(), _stream(stream))
+    _check("treegraft_grow_step", st)
+    return frontier

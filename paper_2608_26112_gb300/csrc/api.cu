@@ -274,6 +274,55 @@ int treegraft_global_prune(const float* score, const int32_t* parent, const int3
                                                                                  : TG_ERR_CUDA;
 }
 
+size_t treegraft_grow_workspace_size(int B, int cap, int m) {
+  if (B < 1 || cap < 1 || cap > TG_MAX_GROW_NODES || m < 1 || m > TG_MAX_TOPK) return 0;
+  return grow_ws_bytes(B, cap, m);
+}
+
+int treegraft_grow_step(int mode, const void* logits, int dtype, int V, int64_t ld, int B, int cap,
+                        int n, int pool_lo, int W, int m, int32_t* parent, int32_t* token,
+                        float* edge, float* score, float* lse_mid, int32_t* frontier, void* ws,
+                        size_t ws_bytes, void* stream) {
+  if (!logits || !parent || !token || !edge || !score || !frontier || !ws) return TG_ERR_INVALID_ARG;
+  if (mode != 0 && mode != 1) return TG_ERR_INVALID_ARG;
+  if (mode == 1 && !lse_mid) return TG_ERR_INVALID_ARG;
+  if (dtype != TG_BF16 && dtype != TG_F32) return TG_ERR_INVALID_ARG;
+  if (B < 1 || cap < 1 || V < 1 || ld < V || n < 1 || n > cap || pool_lo < 0 || pool_lo >= n ||
+      W < 1 || m < 1 || m > V)
+    return TG_ERR_INVALID_ARG;
+  if ((long long)n + (long long)std::min(W, n - pool_lo) * m > (long long)cap)
+    return TG_ERR_INVALID_ARG;  // the children would not fit the tree's capacity
+  if (cap > TG_MAX_GROW_NODES || m > TG_MAX_TOPK || V > (dtype == TG_BF16 ? 262144 : 131072) ||
+      (long long)B * cap > (1ll << 30))
+    return TG_ERR_UNSUPPORTED;
+  if (ws_bytes < grow_ws_bytes(B, cap, m) || !aligned16(ws)) return TG_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(logits) & (dtype == TG_BF16 ? 1 : 3)) != 0)
+    return TG_ERR_INVALID_ARG;  // elements must sit at their natural alignment
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  GrowArgs a;
+  a.mode = mode;
+  a.logits = logits;
+  a.is_bf16 = dtype == TG_BF16;
+  a.V = V;
+  a.ld = ld;
+  a.B = B;
+  a.cap = cap;
+  a.n = n;
+  a.pool_lo = pool_lo;
+  a.W = W;
+  a.m = m;
+  a.parent = parent;
+  a.token = token;
+  a.edge = edge;
+  a.score = score;
+  a.lse_mid = lse_mid;
+  a.frontier = frontier;
+  a.status = st;
+  grow_ws_carve(a, ws, B, cap, m);
+  return launch_grow_step(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK : TG_ERR_CUDA;
+}
+
 int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld, const int32_t* token,
                      const int32_t* parent, const int32_t* node_off, int B, int max_nodes,
                      int n_total, int path_cap, int32_t* path, int32_t* accept_len,

@@ -105,6 +105,32 @@ struct PruneArgs {
 };
 cudaError_t launch_global_prune(const PruneArgs& a, cudaStream_t s);
 
+struct GrowArgs {
+  int mode;  // 0 small-drafter step, 1 middle-drafter step
+  const void* logits;
+  int is_bf16;
+  int V;
+  int64_t ld;
+  int B, cap, n, pool_lo, W, m;
+  int32_t* parent;
+  int32_t* token;
+  float* edge;
+  float* score;
+  float* lse_mid;
+  int32_t* frontier;
+  // workspace (grow_ws_carve)
+  int32_t* ws_row;
+  float* ws_ps;
+  float* ws_lse;
+  int32_t* ws_tok;
+  float* ws_lp;
+  float* ws_sc;
+  int* status;
+};
+size_t grow_ws_bytes(int B, int cap, int m);
+void grow_ws_carve(GrowArgs& a, void* ws, int B, int cap, int m);
+cudaError_t launch_grow_step(const GrowArgs& a, cudaStream_t s);
+
 int device_sm_count();
 // device address of the per-device status word (nullptr on failure)
 int* status_word_ptr();

@@ -140,3 +140,30 @@ def test_global_prune_rejects_bad_args_on_host(lib):
     assert call(path_cap=0) == 1
     assert call(n_total=101) == 1                # more nodes than B * max_nodes
     assert call(max_nodes=2000, n_total=2000) == 2
+
+
+def test_grow_step_rejects_bad_args_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    ws_need = lib.treegraft_grow_workspace_size(2, 64, 4)
+    assert ws_need > 0
+    assert lib.treegraft_grow_workspace_size(2, 2000, 4) == 0      # beyond TG_MAX_GROW_NODES
+    assert lib.treegraft_grow_workspace_size(2, 64, 33) == 0       # beyond TG_MAX_TOPK
+
+    def call(mode=0, dtype=0, V=100, ld=100, B=2, cap=64, n=11, pool_lo=1, W=4, m=4,
+             lse=fake, logits=fake, ws_bytes=None):
+        return lib.treegraft_grow_step(mode, logits, dtype, V, ld, B, cap, n, pool_lo, W, m, fake,
+                                       fake, fake, fake, lse, fake, fake,
+                                       ws_need if ws_bytes is None else ws_bytes, NULL)
+    assert call(logits=NULL) == 1
+    assert call(mode=2) == 1
+    assert call(mode=1, lse=NULL) == 1          # a middle step caches the log-sum-exp
+    assert call(dtype=5) == 1
+    assert call(ld=99) == 1
+    assert call(n=0) == 1
+    assert call(pool_lo=11) == 1                # empty candidate pool
+    assert call(m=101) == 1                     # more children than tokens
+    assert call(n=60) == 1                      # 60 + 4 * 4 children exceed the capacity
+    assert call(ws_bytes=ws_need - 1) == 1
+    assert call(cap=2000, n=11) == 2            # beyond TG_MAX_GROW_NODES
+    assert call(m=33, V=100, cap=1024) == 2     # beyond TG_MAX_TOPK
+    assert call(logits=ctypes.c_void_p(0x1001)) == 1  # misaligned bf16 elements
