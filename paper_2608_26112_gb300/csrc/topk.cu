@@ -3,35 +3,30 @@
 // Algorithms 1 and 2), one HBM pass over the logits.
 //
 // Grid (C, rows) with clusters of C CTAs along x: the C CTAs of a cluster
-// split one row.  Each CTA
-//   1. stages its chunk in registers and takes per-thread (max, sum of
-//      exp(x - max)) - packed bf16x2 max, one exp per element - merged per
-//      warp with shuffles;
-//   2. sorts the 256 thread maxima per warp; after one barrier each of the
-//      top-k lanes of every warp counts, by binary search in the eight
-//      sorted lists, how many maxima reach its own value, and the largest
-//      value with a count >= k is the threshold t = the k-th largest thread
-//      maximum.  At least k elements reach t, and only threads whose max
-//      reaches t can hold elements that do, so candidates are collected by a
-//      handful of threads only, which visit just the 16-byte vectors whose
-//      packed max reaches t;
-//   3. ranks the candidates by 64-bit keys (value desc, token asc - exact
-//      on ties) by counting larger keys.  Heavily tied chunks can overflow
-//      the candidate buffer; they fall back to an exact key threshold (the
-//      k-th largest per-thread (max, first position) key), which bounds the
-//      candidates by 64 * k;
-//   4. the ranking threads store the chunk's top-k (descending) straight
-//      into the cluster leader's shared memory (DSMEM), each warp adds its
-//      (max, sum), and the cluster meets one barrier.
-// In the leader every received key finds its row rank as its index in its
-// own sorted list plus, by binary search, the number of larger keys in each
-// other list; the k keys of rank < k write the outputs, and their warps fold
-// the C * 8 (max, sum) pairs into the lse.  No global scratch and no second
-// launch.
-//
-// These kernels are latency-bound, and several CTAs share an SM: the code
-// keeps dependency chains short and the executed code small (rare paths are
-// rolled loops), so the instruction cache holds the hot path.
+// split one row.  The selection uses no block barrier, only three phases of
+// the cluster barrier:
+//   0. every CTA stages its chunk in registers (eight 16-byte loads per
+//      thread, all in flight at once) and takes its thread maxima; each warp
+//      finds its top r lane maxima (r = ceil(k / (8 C)), so the row pushes at
+//      least k values) and stores them into EVERY CTA of the cluster (DSMEM);
+//   1. while the other CTAs finish, each thread takes the sum of exp(x - max)
+//      over its elements (packed bf16x2 max, one exp per element), each warp
+//      folds its lanes' (max, sum) with one exponential per lane and pushes
+//      the pair to the leader.  After the barrier every
+//      warp holds the same 8 C r pushed maxima and takes their k-th largest
+//      T: k distinct elements of the row reach T, so the row's top-k all do.
+//      Only threads whose max reaches T hold elements that do; they visit
+//      the 16-byte vectors whose packed max reaches T and push those
+//      elements' 64-bit keys (value desc, token asc - exact on ties) into the
+//      leader's candidate buffer (DSMEM atomics);
+//   2. the leader ranks the few candidates by counting larger keys, folds
+//      the C * 8 (max, sum) pairs into the lse, and writes token, logprob =
+//      x - lse and score = fp32(parent_score + logprob).  A tie-heavy row that
+//      overflows the candidate buffer is ranked exactly by the leader alone
+//      from global memory (k rounds of a block-wide key max) - slow, rare.
+// No global scratch and no second launch.  The kernels are latency-bound
+// after the load, so the code keeps dependency chains short and the
+// executed code small (rare paths are rolled loops).
 #include <cooperative_groups.h>
 
 #include "launch.h"
@@ -42,91 +37,97 @@ namespace cg = cooperative_groups;
 namespace tg {
 namespace {
 
-constexpr int kMaxK = 32;
-constexpr int kCandMax = 2048;  // >= 64 elements/thread * kMaxK
+constexpr int kMaxK = 32;  // TG_MAX_TOPK
 constexpr int kMaxCluster = 16;
-static_assert(kCandMax >= kScanVecs * 8 * kMaxK, "exact fallback must fit the buffer");
+constexpr int kMaxPush = 128;   // pushed lane maxima per row: 8 C r <= 128
+// r = ceil(k / (8 C)) <= 4 lane maxima per warp give 8 C r >= k pushed values
+static_assert(kMaxK <= 8 * 4 && 8 * kMaxCluster <= kMaxPush, "push sizes");
+constexpr int kCandMax = 2048;  // the leader's candidate buffer
 
 struct TopkSmem {
-  uint64_t cand[kCandMax];
-  uint64_t recv_top[kMaxCluster * kMaxK];  // leader only: each CTA's sorted top-k
-  float recv_m[kMaxCluster * 8];           // leader only: each warp's (max, sum)
+  uint64_t cand[kCandMax];        // leader: candidate keys of the whole row
+  float push_v[kMaxPush];         // every CTA: the row's pushed lane maxima
+  float recv_m[kMaxCluster * 8];  // leader: each warp's (max, sum)
   float recv_s[kMaxCluster * 8];
-  float warp_v[8 * 32];  // each warp's 32 thread maxima, sorted descending
-  uint64_t warp_k[8 * kMaxK];
-  uint64_t thr_key;
-  uint32_t thr_ord;
-  int ncand;
+  uint64_t red_k[8];              // leader fallback: block reduction
+  int ncand;                      // leader: candidate count
 };
 
-// Entries >= x in the eight descending 32-float lists L[w * 32 ..]: eight
-// branch-free binary searches run in lockstep (5 halving steps and a final
-// probe), so each step issues eight independent shared loads.
-__device__ __forceinline__ int count_ge_8x32(const float* L, float x) {
-  int pos[8];
+// (max, sum of exp(x - max)) of the 32 lanes' pairs, in every lane: the max
+// by one warp-wide integer max, one exponential per lane, a shuffle sum.
+__device__ __forceinline__ void warp_lse_pair(float& m, float& s) {
+  const float NEG_INF = __int_as_float(0xff800000);
+  const float M = unord_f32(__reduce_max_sync(0xffffffffu, ord_f32(m)));
+  float t = (m == NEG_INF) ? 0.f : s * ex2((m - M) * kLog2e);
 #pragma unroll
-  for (int w = 0; w < 8; ++w) pos[w] = 0;
-#pragma unroll
-  for (int step = 16; step > 0; step >>= 1)
-#pragma unroll
-    for (int w = 0; w < 8; ++w) pos[w] += (L[w * 32 + pos[w] + step - 1] >= x) ? step : 0;
-  int cnt = 0;
-#pragma unroll
-  for (int w = 0; w < 8; ++w) cnt += pos[w] + ((L[w * 32 + pos[w]] >= x) ? 1 : 0);
-  return cnt;
+  for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+  m = M;
+  s = t;
 }
 
-// Keys > x in the C descending lists of n <= 32 keys at L[c * n ..], list
-// `skip` excluded: the C binary searches run in lockstep.
-__device__ __forceinline__ int count_gt_lists(const uint64_t* L, int C, int n, int skip,
-                                              uint64_t x) {
-  int pos[kMaxCluster];
-#pragma unroll
-  for (int c = 0; c < kMaxCluster; ++c) pos[c] = 0;
-#pragma unroll
-  for (int step = 16; step > 0; step >>= 1)
-#pragma unroll
-    for (int c = 0; c < kMaxCluster; ++c) {
-      const int i = pos[c] + step - 1;
-      if (c < C && i < n && L[c * n + i] > x) pos[c] += step;
-    }
-  int cnt = 0;
-#pragma unroll
-  for (int c = 0; c < kMaxCluster; ++c)
-    if (c < C && c != skip) cnt += pos[c] + ((pos[c] < n && L[c * n + pos[c]] > x) ? 1 : 0);
-  return cnt;
-}
-
-// descending bitonic sort of one value per lane; lane j ends with the j-th largest
-template <typename K>
-__device__ __forceinline__ K warp_sort_desc(K x) {
+// r rounds of warp-wide max extraction: lane i < r ends with the i-th
+// largest of the 32 lane values (each round pops one lane holding the max;
+// ties are popped one at a time, lowest lane first).
+__device__ __forceinline__ float warp_top_r(float x, int r) {
   const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int size = 2; size <= 32; size <<= 1) {
-#pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      const K y = __shfl_xor_sync(0xffffffffu, x, stride);
-      const bool take_max = (((lane & stride) == 0) == ((lane & size) == 0));
-      x = take_max ? (x > y ? x : y) : (x < y ? x : y);
+  float out = __int_as_float(0xff800000);
+  uint32_t h = ord_f32(x);
+  for (int i = 0; i < r; ++i) {
+    const uint32_t mx = __reduce_max_sync(0xffffffffu, h);
+    const uint32_t who = __ffs(__ballot_sync(0xffffffffu, h == mx)) - 1;
+    if (lane == i) out = unord_f32(mx);
+    if (lane == (int)who) h = 0u;  // below every ordered value (ord(-inf) > 0)
+  }
+  return out;
+}
+
+// k-th largest (with multiplicity) of the n <= 128 values at v[]: each lane
+// sorts its 4 values, then rounds of warp-wide max extraction count them
+// down.  Every lane returns the same value.
+__device__ __forceinline__ float kth_largest_128(const float* v, int n, int k) {
+  const int lane = threadIdx.x & 31;
+  const float NEG_INF = __int_as_float(0xff800000);
+  float a0 = lane < n ? v[lane] : NEG_INF;
+  float a1 = lane + 32 < n ? v[lane + 32] : NEG_INF;
+  float a2 = lane + 64 < n ? v[lane + 64] : NEG_INF;
+  float a3 = lane + 96 < n ? v[lane + 96] : NEG_INF;
+  auto cas = [](float& x, float& y) {
+    const float hi = fmaxf(x, y), lo = fminf(x, y);
+    x = hi;
+    y = lo;
+  };
+  cas(a0, a1);
+  cas(a2, a3);
+  cas(a0, a2);
+  cas(a1, a3);
+  cas(a1, a2);
+  int cnt = 0;
+  for (int round = 0; round < kMaxPush; ++round) {  // ends after at most k rounds
+    const uint32_t h = ord_f32(a0);
+    const uint32_t mx = __reduce_max_sync(0xffffffffu, h);
+    const bool mine = h == mx;
+    cnt += __popc(__ballot_sync(0xffffffffu, mine));
+    if (cnt >= k) return unord_f32(mx);
+    if (mine) {
+      a0 = a1;
+      a1 = a2;
+      a2 = a3;
+      a3 = NEG_INF;
     }
   }
-  return x;
+  return NEG_INF;
 }
 
-__device__ __forceinline__ void push_cand(TopkSmem& sm, uint64_t key) {
-  const int slot = atomicAdd(&sm.ncand, 1);
-  if (slot < kCandMax) sm.cand[slot] = key;
-}
-
-// Elements >= tv of this thread's chunk into the candidate buffer.  Only the
-// vectors whose packed max reaches tv are visited (typically one).
+// Elements >= tv of this thread's chunk into the leader's candidate buffer
+// (DSMEM atomics for the slots).  Only the vectors whose packed max reaches
+// tv are visited (typically one).
 template <typename T>
-__device__ __forceinline__ void collect_candidates(const uint4 (&buf)[kScanVecs], int c0, int c1,
-                                                   float tv, TopkSmem& sm) {
+__device__ __forceinline__ void push_candidates(const uint4 (&buf)[kScanVecs], int c0, int c1,
+                                                float tv, TopkSmem* lead) {
   constexpr int VW = ScanTraits<T>::kVW;
   uint32_t hit = 0;
   if constexpr (VW == 8) {
-    // tv is a thread max, so it is exactly representable in bf16
+    // tv is an element value, so it is exactly representable in bf16
     const __nv_bfloat162 tv2 = __float2bfloat162_rn(tv);
 #pragma unroll
     for (int i = 0; i < kScanVecs; ++i) {
@@ -171,56 +172,41 @@ __device__ __forceinline__ void collect_candidates(const uint4 (&buf)[kScanVecs]
       const uint32_t w = vec_word(q, VW == 8 ? (j >> 1) : j);
       const float v = VW == 8 ? ((j & 1) ? bf16_hi(w) : bf16_lo(w)) : __uint_as_float(w);
       const int pos = scan_pos(c0, i, j, VW);
-      if (pos < c1) push_cand(sm, make_key(v, (uint32_t)pos));
+      if (pos < c1) {
+        const int slot = atomicAdd(&lead->ncand, 1);
+        if (slot < kCandMax) lead->cand[slot] = make_key(v, (uint32_t)pos);
+      }
     }
   }
 }
 
-// Heavy ties (the candidate buffer overflowed): exact key threshold = the
-// k-th largest per-thread (max, first position) key; candidates are the
-// elements whose key reaches it (at most 64 * k).  The chunk is re-read from
-// global memory in rolled loops: this path is rare and stays out of the hot
-// code.  Called by every thread of the CTA; returns the candidate count.
+// Leader only, when the candidate buffer overflowed (heavy ties): the row's
+// exact top-k by k rounds of a block-wide max over the keys below the last
+// one found, read from global memory.  Returns in smem cand[0..k).
 template <typename T>
-__device__ __noinline__ int tie_fallback(const T* __restrict__ rowp, int c0, int c1, int k,
-                                         float tmax, TopkSmem& sm) {
-  constexpr int VW = ScanTraits<T>::kVW;
+__device__ __noinline__ void exact_topk_fallback(const T* __restrict__ rowp, int V, int k,
+                                                 TopkSmem& sm) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  __syncthreads();  // every thread has read ncand before it is reset below
-  int fp = 0x7FFFFFFF;
+  uint64_t last = ~0ull;
 #pragma unroll 1
-  for (int e = 0; e < kScanVecs * VW && fp == 0x7FFFFFFF; ++e) {
-    const int pos = scan_pos(c0, e / VW, e % VW, VW);
-    if (pos < c1 && load_elem<T>(rowp, pos) == tmax) fp = pos;
-  }
-  const uint64_t tk = (fp == 0x7FFFFFFF) ? 0ull : make_key(tmax, (uint32_t)fp);
-  const uint64_t sk = warp_sort_desc<uint64_t>(tk);
-  if (lane < k) sm.warp_k[warp * k + lane] = sk;
-  if (tid == 0) {
-    sm.thr_key = 0ull;
-    sm.ncand = 0;
-  }
-  __syncthreads();
-  if (tid < 8 * k) {
-    const uint64_t mine = sm.warp_k[tid];
-    int rank = 0;
-    for (int i = 0; i < 8 * k; ++i) rank += (sm.warp_k[i] > mine) ? 1 : 0;
-    if (mine != 0ull && rank == k - 1) sm.thr_key = mine;
-  }
-  __syncthreads();
-  const uint64_t thr = sm.thr_key;
-  if (tk >= thr && tk != 0ull) {
+  for (int r = 0; r < k; ++r) {
+    uint64_t best = 0ull;
 #pragma unroll 1
-    for (int e = 0; e < kScanVecs * VW; ++e) {
-      const int pos = scan_pos(c0, e / VW, e % VW, VW);
-      if (pos < c1) {
-        const uint64_t key = make_key(load_elem<T>(rowp, pos), (uint32_t)pos);
-        if (key >= thr) push_cand(sm, key);
-      }
+    for (int pos = tid; pos < V; pos += kScanThreads) {
+      const uint64_t key = make_key(load_elem<T>(rowp, pos), (uint32_t)pos);
+      if (key < last && key > best) best = key;
     }
+    best = warp_max_u64(best);
+    if (lane == 0) sm.red_k[warp] = best;
+    __syncthreads();
+    best = sm.red_k[0];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) best = sm.red_k[w] > best ? sm.red_k[w] : best;
+    __syncthreads();
+    if (tid == 0) sm.cand[r] = best;
+    last = best;
   }
   __syncthreads();
-  return min(sm.ncand, kCandMax);
 }
 
 template <typename T, bool kAligned>
@@ -245,7 +231,9 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
     if (crank == 0 && tid == 0) raise_status(a.status, kStIndex);
     return;
   }
-  cluster_arrive_relaxed();
+  if (crank == 0 && tid == 0) sm.ncand = 0;
+  // phase 0: the leader's counter is initialised before any CTA can push
+  cluster_arrive_release();
   // the leader's threads fetch the parent's path score now, while the
   // logits are in flight (one broadcast request per warp)
   float parent_score = 0.f;
@@ -257,75 +245,52 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
 
   uint4 buf[kScanVecs];
   scan_load<T, kAligned>(rowp, c0, c1, buf);
-  if (tid == 0) {
-    sm.ncand = 0;
-    sm.thr_ord = 0u;
-  }
-
-  // 1. per-thread max and exp-sum, warp-combined
   const float tmax = scan_thread_max<T>(buf);
-  float m = tmax, s = scan_thread_sumexp<T>(buf, tmax);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
-    lse_merge(m, s, m2, s2);
-  }
-  // 2. value threshold: the k-th largest of the 256 thread maxima.  It is
-  //    among the top k of some warp's sorted list; each such entry counts
-  //    the maxima >= itself in all eight lists, and the largest entry with
-  //    a count >= k is the k-th largest.
-  const float sv = warp_sort_desc<float>(tmax);
-  sm.warp_v[warp * 32 + lane] = sv;
-  __syncthreads();
-  if (lane < k && count_ge_8x32(sm.warp_v, sv) >= k) atomicMax(&sm.thr_ord, ord_f32(sv));
-  __syncthreads();
-  const float tv = unord_f32(sm.thr_ord);
-  // 3. candidates (only threads whose max reaches the threshold have any)
-  if (tmax >= tv) collect_candidates<T>(buf, c0, c1, tv, sm);
-  __syncthreads();
-  int nc = sm.ncand;
-  if (nc > kCandMax) nc = tie_fallback<T>(rowp, c0, c1, k, tmax, sm);
-
-  // 4. rank the candidates and store the chunk's top-k (descending) straight
-  //    into the leader's receive slots; slots past the candidates get 0
-  cluster_wait();  // every CTA of the cluster is running: DSMEM is addressable
+  // each warp's top rp lane maxima go to every CTA of the cluster
+  const int rp = min(4, (k + 8 * C - 1) / (8 * C));
+  const int npush = 8 * C * rp;
+  const float top = warp_top_r(tmax, rp);
+  cluster_wait_acquire();
   TopkSmem* lead = cluster.map_shared_rank(&sm, 0);
-  uint64_t* dst = lead->recv_top + crank * k;
-  for (int i = tid; i < nc; i += kScanThreads) {
-    const uint64_t mine = sm.cand[i];
-    int rank = 0;
-#pragma unroll 4
-    for (int j = 0; j < nc; ++j) rank += (sm.cand[j] > mine) ? 1 : 0;
-    if (rank < k) dst[rank] = mine;
+  if (lane < rp) {
+    const int slot = (crank * 8 + warp) * rp + lane;
+    for (int c = 0; c < C; ++c) cluster.map_shared_rank(&sm, c)->push_v[slot] = top;
   }
-  if (tid >= nc && tid < k) dst[tid] = 0ull;
+  // phase 1: the pushed maxima become visible; the exp-sum runs while the
+  // other CTAs finish their loads
+  cluster_arrive_release();
+  float m = tmax, s = scan_thread_sumexp<T>(buf, tmax);
+  warp_lse_pair(m, s);
   if (lane == 0) {
     lead->recv_m[crank * 8 + warp] = m;
     lead->recv_s[crank * 8 + warp] = s;
   }
-  cluster.sync();
+  cluster_wait_acquire();
+  const float tv = kth_largest_128(sm.push_v, npush, k);
+  if (tmax >= tv) push_candidates<T>(buf, c0, c1, tv, lead);
+  // phase 2: every candidate and (max, sum) has reached the leader
+  cluster_arrive_release();
+  cluster_wait_acquire();
   if (crank != 0) return;
 
-  // ---- leader: key t (list c = t / k, index j = t % k) has row rank
-  // j + the number of larger keys in the other lists (keys are unique; empty
-  // slots are 0 and never reach rank k, as the row has >= k real keys)
-  const int ck = C * k;
-  if (warp * 32 >= ck) return;
+  // ---- leader: lse and the row's top-k from the candidates
+  const int nc = sm.ncand;
+  if (nc > kCandMax) exact_topk_fallback<T>(rowp, V, k, sm);
+  const int nr = nc > kCandMax ? k : nc;  // keys to rank; the fallback's are already in order
+  if (warp * 32 >= nr) return;
   float M = NEG_INF, S = 0.f;
   for (int i = lane; i < C * 8; i += 32) lse_merge(M, S, sm.recv_m[i], sm.recv_s[i]);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, M, o);
-    const float s2 = __shfl_xor_sync(0xffffffffu, S, o);
-    lse_merge(M, S, m2, s2);
-  }
+  warp_lse_pair(M, S);
   const float lse = (M == NEG_INF) ? M : M + log2f(S) * kLn2;
-  for (int t = tid; t < ck; t += kScanThreads) {
-    const uint64_t key = sm.recv_top[t];
-    const int c = t / k;
-    const int rank = t - c * k + count_gt_lists(sm.recv_top, C, k, c, key);
-    if (key != 0ull && rank < k) {
+  for (int t = tid; t < nr; t += kScanThreads) {
+    const uint64_t key = sm.cand[t];
+    int rank = t;
+    if (nc <= kCandMax) {
+      rank = 0;
+#pragma unroll 4
+      for (int j = 0; j < nr; ++j) rank += (sm.cand[j] > key) ? 1 : 0;
+    }
+    if (rank < k) {
       const float v = key_value(key);
       const float lp = (lse == NEG_INF) ? lse : (v - lse);
       const size_t o = (size_t)row * k + rank;
