@@ -170,29 +170,6 @@ __device__ __forceinline__ float scan_thread_max<float>(const uint4 (&buf)[kScan
   return m;
 }
 
-// 2^y for y <= 0, two at a time, on the FMA pipe instead of the MUFU unit:
-// y = j + f with j = rint(y) and |f| <= 1/2; 2^f comes from a degree-4
-// polynomial (a weighted least-squares fit of 2^f on [-1/2, 1/2] made for
-// this kernel: max relative error 2.7e-6 when evaluated in fp32 Horner form)
-// and 2^j is added into the exponent field.  Adding 1.5 * 2^23 rounds y to
-// an integer in the low mantissa bits of t, and (bits(t) << 23) is exactly
-// j << 23 modulo 2^32.  y is clamped at -126 so the exponent never wraps;
-// such terms are below fp32 resolution of a sum that holds 2^0 = 1.
-__device__ __forceinline__ float2 exp2_poly2(float2 y) {
-  y.x = fmaxf(y.x, -126.f);
-  y.y = fmaxf(y.y, -126.f);
-  const float2 t = __fadd2_rn(y, make_float2(12582912.f, 12582912.f));
-  const float2 j = __fadd2_rn(t, make_float2(-12582912.f, -12582912.f));
-  const float2 f = __ffma2_rn(j, make_float2(-1.f, -1.f), y);
-  float2 p = __ffma2_rn(make_float2(0.009570101276040077f, 0.009570101276040077f), f,
-                        make_float2(0.05591785907745361f, 0.05591785907745361f));
-  p = __ffma2_rn(p, f, make_float2(0.240247443318367f, 0.240247443318367f));
-  p = __ffma2_rn(p, f, make_float2(0.6931217908859253f, 0.6931217908859253f));
-  p = __ffma2_rn(p, f, make_float2(0.9999992847442627f, 0.9999992847442627f));
-  return make_float2(__uint_as_float(__float_as_uint(p.x) + (__float_as_uint(t.x) << 23)),
-                     __uint_as_float(__float_as_uint(p.y) + (__float_as_uint(t.y) << 23)));
-}
-
 // elements 2w, 2w+1 of a 16-byte vector as a float pair
 template <typename T>
 __device__ __forceinline__ float2 vec_pair(const uint4& v, int w);
@@ -206,12 +183,10 @@ __device__ __forceinline__ float2 vec_pair<float>(const uint4& v, int w) {
   return make_float2(__uint_as_float(vec_word(v, 2 * w)), __uint_as_float(vec_word(v, 2 * w + 1)));
 }
 
-// Vectors [0, kMufuVecs) take their exponentials on the MUFU unit, the rest
-// on the FMA pipe (exp2_poly2): MUFU throughput is an eighth of the issue
-// rate, so 3 of 8 vectors on the FMA pipe balances the two.
-constexpr int kMufuVecs = 5;
-
-// sum_t 2^((x_t - m) * log2 e) over this thread's elements, m = its max
+// sum_t 2^((x_t - m) * log2 e) over this thread's elements, m = its max, on
+// the MUFU unit (one ex2 per element; after the load the scan kernels are
+// bound by latency, not by MUFU throughput, and a share of polynomial
+// exponentials on the FMA pipe measured slower)
 template <typename T>
 __device__ __forceinline__ float scan_thread_sumexp(const uint4 (&buf)[kScanVecs], float m) {
   if (m == __int_as_float(0xff800000)) return 0.f;
@@ -224,11 +199,8 @@ __device__ __forceinline__ float scan_thread_sumexp(const uint4 (&buf)[kScanVecs
 #pragma unroll
     for (int w = 0; w < VW / 2; ++w) {
       const float2 y = __ffma2_rn(vec_pair<T>(buf[i], w), l2e, nb);
-      if (i < kMufuVecs) {
-        acc0 = __fadd2_rn(acc0, make_float2(ex2(y.x), ex2(y.y)));
-      } else {
-        acc1 = __fadd2_rn(acc1, exp2_poly2(y));
-      }
+      const float2 e = make_float2(ex2(y.x), ex2(y.y));
+      if (i & 1) acc1 = __fadd2_rn(acc1, e); else acc0 = __fadd2_rn(acc0, e);
     }
   return (acc0.x + acc0.y) + (acc1.x + acc1.y);
 }
