@@ -216,6 +216,123 @@ def prune_timing(R, seed, dev, stream, reps):
             "in_step": False, "note": "Algorithm 3 on the pre-pruning tree, latency-bound"}
 
 
+EXTRA_CONFIGS = ["llama3-70b-verify", "graft-mha"]
+
+
+def config_timing(name, seed, dev, stream, n_sets=2, seconds=0.15):
+    """The step's four kernels on another synthetic workload, timed alone
+    (not part of the headline step): per-kernel launch time over n_sets
+    rotating input sets, attention FLOP/s against the bf16 tensor peak and
+    bytes/s against the HBM peak.  For the Llama-3-70B-shaped verify batch
+    (4 trees of 128 nodes, prefix 8192, GQA 64/8) the attention is
+    tensor-bound (137 GFLOP per launch)."""
+    import numpy as np
+    import torch
+    import paper_2608_26112_gb300 as tg
+    from paper_2608_26112_gb300 import synth
+
+    def bf(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    def t(a):
+        return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+    sets = []
+    for r in range(n_sets):
+        wl = synth.make_workload(name, seed=seed + r)
+        sh = wl["shape"]
+        rng = synth.make_rng(40_000 + seed + r)
+        lg = wl["logits"]
+        bf16 = lg.dtype == np.uint16
+        tl = synth.normal_f32(rng, lg.shape, 3.0)
+        synth.plant_child_bump(rng, tl, wl["parent"], wl["token"], np.arange(len(wl["parent"])))
+        target = synth.f32_to_bf16_bits(tl) if bf16 else tl
+        node_off = wl["node_off"]
+        B = len(node_off) - 1
+        mx = int(np.max(np.diff(node_off)))
+        n_total = len(wl["parent"])
+        d = dict(q=bf(wl["q"]), k=bf(wl["k_cache"]), v=bf(wl["v_cache"]),
+                 prefix_len=t(wl["prefix_len"]), parent=t(wl["parent"]), token=t(wl["token"]),
+                 node_off=t(node_off), logits=bf(lg) if bf16 else t(lg),
+                 target=bf(target) if bf16 else t(target), parent_score=t(wl["parent_score"]),
+                 weak_edge=t(wl["weak_edge"]), visited=t(wl["visited"]), strong=t(wl["strong_lp"]))
+        k, N = sh["k"], sh["N"]
+        o = dict(o=torch.empty_like(d["q"]),
+                 tok=torch.empty(n_total, k, dtype=torch.int32, device=dev),
+                 lp=torch.empty(n_total, k, dtype=torch.float32, device=dev),
+                 sc=torch.empty(n_total, k, dtype=torch.float32, device=dev),
+                 edge=torch.empty(n_total, dtype=torch.float32, device=dev),
+                 score=torch.empty(n_total, dtype=torch.float32, device=dev),
+                 sel=torch.empty(B, N, dtype=torch.int32, device=dev),
+                 nsel=torch.empty(B, dtype=torch.int32, device=dev),
+                 path=torch.empty(B, mx, dtype=torch.int32, device=dev),
+                 alen=torch.empty(B, dtype=torch.int32, device=dev),
+                 bonus=torch.empty(B, dtype=torch.int32, device=dev),
+                 ws=tg.accept_workspace(B, n_total, dev),
+                 attn_ws=torch.zeros(max(16, tg.tree_attn_workspace_size(
+                     B, mx, sh["Hq"], sh["Hkv"], sh["D"])), dtype=torch.uint8, device=dev))
+        sets.append((wl, d, o, mx))
+    wl, _, _, mx = sets[0]
+    sh = wl["shape"]
+
+    def run(kname, d, o, mx):
+        if kname == "tree_attn":
+            tg.tree_attn(d["q"], d["k"], d["v"], d["prefix_len"], d["parent"], d["node_off"], mx,
+                         out=o["o"], ws=o["attn_ws"], stream=stream)
+        elif kname == "expand_topk":
+            tg.expand_topk(d["logits"], d["parent_score"], sh["k"], out=(o["tok"], o["lp"], o["sc"]),
+                           stream=stream)
+        elif kname == "rescore_select":
+            tg.rescore_select(d["weak_edge"], d["strong"], d["parent"], d["token"], d["visited"],
+                              d["node_off"], mx, sh["N"],
+                              out=(o["edge"], o["score"], o["sel"], o["nsel"]), stream=stream)
+        else:
+            tg.accept(d["target"], d["token"], d["parent"], d["node_off"], mx, mx, o["ws"],
+                      out=(o["path"], o["alen"], o["bonus"]), stream=stream)
+
+    with torch.cuda.stream(stream):
+        for _, d, o, m_ in sets:
+            for kname in KERNELS:
+                run(kname, d, o, m_)
+    stream.synchronize()
+    assert tg.last_device_status(stream) == 0
+    # algorithmic costs of set 0
+    parent, node_off = wl["parent"], wl["node_off"]
+    B = len(node_off) - 1
+    Hq, Hkv, D, V = sh["Hq"], sh["Hkv"], sh["D"], sh["V"]
+    elem = 2 if wl["logits"].dtype == np.uint16 else 4
+    keys, kv_bytes = 0, 0
+    for b in range(B):
+        lo, hi = int(node_off[b]), int(node_off[b + 1])
+        P = int(wl["prefix_len"][b])
+        depth = [0] * (hi - lo)
+        for v in range(1, hi - lo):
+            depth[v] = depth[parent[lo + v]] + 1
+        keys += sum(P + dd + 1 for dd in depth)
+        kv_bytes += 2 * (P + hi - lo) * Hkv * D * 2
+    n_total = len(parent)
+    costs = dict(tree_attn=(kv_bytes + 2 * n_total * Hq * D * 2, 4 * Hq * D * keys),
+                 expand_topk=(n_total * V * elem, 0), accept=(n_total * V * elem, 0),
+                 rescore_select=(n_total * 17, 0))
+    pk, _ = peaks()
+    out = {}
+    for kname in KERNELS:
+        g = capture(lambda kname=kname: [run(kname, d, o, m_) for _, d, o, m_ in sets], stream)
+        g.replay()
+        t1 = time_graph(g, 3, stream) / (3 * n_sets)
+        reps = max(3, min(2000, int(seconds / max(t1 * n_sets, 1e-7))))
+        tk = time_graph(g, reps, stream) / (reps * n_sets)
+        b_, f_ = costs[kname]
+        ent = {"us": tk * 1e6, "bytes": b_, "GBps": b_ / tk / 1e9, "hbm_frac": b_ / tk / 1e9 / pk["hbm_gbs"]}
+        if f_:
+            ent["TFLOPs"] = f_ / tk / 1e12
+            ent["tensor_frac"] = f_ / tk / 1e12 / pk["bf16_tflops"]
+            ent["roofline_frac"] = max(b_ / (pk["hbm_gbs"] * 1e9), f_ / (pk["bf16_tflops"] * 1e12)) / tk
+        out[kname] = ent
+    return {"shape": {k_: v_ for k_, v_ in sh.items() if k_ in ("B", "P", "n", "Hq", "Hkv", "D", "V", "k", "N")},
+            "kernels": out, "sets": n_sets}
+
+
 GROW_SCHEDULE = [1, 0, 1, 0, 1]
 
 
@@ -546,6 +663,8 @@ def ours_arm(args):
             kt[name] = time_graph(g, kreps, stream) / (kreps * R)
         prune = prune_timing(R, rank_seed(args.seed, rank), dev, stream, kreps)
         grow = grow_timing(rank_seed(args.seed, rank), dev, stream, kreps)
+        extra = {nm: config_timing(nm, rank_seed(args.seed, rank), dev, stream)
+                 for nm in EXTRA_CONFIGS}
     assert tg.last_device_status(stream) == 0
     t_max = max_over_ranks(t_steps, world)
     steps_per_s = job_throughput(world, K, t_max)
@@ -588,7 +707,7 @@ def ours_arm(args):
                        "l2": f"{R} rotating input sets, ~{R * 40} MB touched per cycle "
                              + ("> 126 MB L2" if R * 40 > 126 else "(fits in L2)"),
                        "parallelism": f"independent sequences per GPU x{world}"},
-            "roofline": roofline, "kernels": kernels, "e2e": e2e,
+            "roofline": roofline, "kernels": kernels, "other_workloads": extra, "e2e": e2e,
             "gpu_launches": K * len(KERNELS), "clocks": clocks.summary()}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         steps_c, sec = run_cpu_oracle(3, 1, 10.0, 30.0)

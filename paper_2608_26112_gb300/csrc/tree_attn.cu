@@ -13,17 +13,22 @@
 // Warp roles (320 threads, one CTA per SM):
 //   warp 0      TMA producer: K and V tiles into a 2-stage ring, Q once;
 //   warp 1      TMEM owner and MMA issuer: S = Q K^T (M=128, N=128, K=D) into
-//               one of two TMEM buffers and O += P V (M=128, N=D, K=128),
-//               bf16 in, fp32 accumulate, completion signalled by
-//               tcgen05.commit on mbarriers.  Pipe order S(0) S(1) PV(0)
-//               S(2) PV(1) ...: S(i+1) runs while the softmax of tile i runs;
+//               one of two TMEM buffers and O += P V (M=128, N=D, K=128) with
+//               P read from TMEM, bf16 in, fp32 accumulate, completion
+//               signalled by tcgen05.commit on mbarriers.  Pipe order S(0)
+//               S(1) PV(0) S(2) PV(1) ...: S(i+1) runs while the softmax of
+//               tile i runs; S(i+2) reuses the buffer of P(i) once PV(i) is
+//               done;
 //   warps 2..9  softmax: two threads per query row (TMEM lane = row), each
 //               owning half of the 128 key columns and half of O's columns.
 //               They read S with tcgen05.ld, apply the ancestor mask from a
 //               per-node bitmask in shared memory, exchange the row max
 //               through shared memory, keep a base-2 online max / sum, write
-//               P as bf16 into the swizzled operand layout, and rescale O in
-//               TMEM when the running max grows.
+//               P as bf16 over the S buffer it came from (tcgen05.st), and
+//               rescale O in TMEM only when the row max grows by more than 8
+//               (base 2) past the reference the tile's P was taken against.
+//               P(i+1) goes to the other TMEM buffer than P(i), so the
+//               softmax never waits for PV(i) unless O has to be rescaled.
 // Split combine: each CTA stages its partial rows (O, max, sum) in shared
 // memory, copies them with coalesced stores into the caller's workspace (L2
 // resident), and after one cluster barrier reduces the S_kv partials of the
@@ -52,8 +57,11 @@ constexpr float kLn2 = 0.6931471805599453f;
 // K and V have their own rings: a K stage is free once its S = Q K^T
 // product is done, a V stage once its PV product is, so the next K tile is
 // requested well before the current PV finishes.
+// PV(j) commits to BAR_O_DONE + (j & 1) (phase j >> 1): with two barriers a
+// waiter that observes PV(j) before P(j + 2) can be produced never finds a
+// barrier two phases ahead, so the softmax may skip waits on PV products.
 enum { BAR_K_FULL = 0, BAR_V_FULL = 2, BAR_K_EMPTY = 4, BAR_V_EMPTY = 6, BAR_Q_FULL = 8,
-       BAR_S_FULL = 9 /* 2 buffers */, BAR_P_FULL = 11, BAR_O_DONE = 12, kNumBars = 13 };
+       BAR_S_FULL = 9 /* 2 buffers */, BAR_P_FULL = 11, BAR_O_DONE = 12 /* 2 */, kNumBars = 14 };
 
 constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
@@ -61,12 +69,10 @@ template <int D>
 struct Layout {
   static constexpr int kQBytes = kBM * D * 2;
   static constexpr int kKVBytes = kBN * D * 2;
-  static constexpr int kPBytes = kBM * kBN * 2;
   static constexpr int kOffQ = 0;
   static constexpr int kOffK = kOffQ + kQBytes;
   static constexpr int kOffV = kOffK + kStages * kKVBytes;
-  static constexpr int kOffP = kOffV + kStages * kKVBytes;
-  static constexpr int kTileEnd = kOffP + kPBytes;
+  static constexpr int kTileEnd = kOffV + kStages * kKVBytes;
   static constexpr int kOffAnc = kTileEnd;                            // (kBM + 1) rows
   static constexpr int kOffPar = align_up(kOffAnc + (kBM + 1) * kAncWords * 4, 16);
   static constexpr int kOffRedMax = align_up(kOffPar + 256 * 4, 16); // [2 parity][2 half][kBM]
@@ -83,7 +89,7 @@ struct Layout {
   static constexpr int kSlabM = kBM * D * 2;  // byte offset of m[] (fp32)
   static constexpr int kSlabL = kSlabM + kBM * 4;  // byte offset of l[] (fp32)
   static_assert(kAlloc <= 227 * 1024, "shared memory budget");
-  static_assert(kOffQ % 1024 == 0 && kOffK % 1024 == 0 && kOffV % 1024 == 0 && kOffP % 1024 == 0,
+  static_assert(kOffQ % 1024 == 0 && kOffK % 1024 == 0 && kOffV % 1024 == 0,
                 "128-byte-swizzled operand tiles need 1024-byte alignment");
   static_assert(kOffBar % 8 == 0 && kOffMisc % 16 == 0, "mbarrier / scalar alignment");
   static_assert(kSlabBytes % 16 == 0 && kSlabM % 16 == 0, "16-byte slab groups");
@@ -246,7 +252,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t q_base = smem_u32(smem + L::kOffQ);
   const uint32_t k_base = smem_u32(smem + L::kOffK);
   const uint32_t v_base = smem_u32(smem + L::kOffV);
-  const uint32_t p_base = smem_u32(smem + L::kOffP);
   const float NEG_INF = __int_as_float(0xff800000);
 
   // the next kernel on the stream may be dispatched now; this one's global
@@ -303,6 +308,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(bar(BAR_Q_FULL), 1);
     mbar_init(bar(BAR_P_FULL), kSoftmaxThreads);
     mbar_init(bar(BAR_O_DONE), 1);
+    mbar_init(bar(BAR_O_DONE + 1), 1);
     fence_mbar_init();
     *bad_flag = 0;
     tma_prefetch_desc(&tm_k);
@@ -379,10 +385,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = mbar_wait(bar(BAR_Q_FULL), 0);
       for (int it = 0; ok && it <= nt; ++it) {
         if (it < nt) {
-          // S buffer it&1 was last read by the softmax of tile it-2, whose
-          // P_FULL phase was awaited before PV(it-2) was issued
+          // S buffer it&1 holds P(it-2): S(it) may overwrite it once PV(it-2)
+          // is done (MMAs with different accumulators are not ordered)
           const int st = it & 1;
           ok = mbar_wait(bar(BAR_K_FULL + st), (it >> 1) & 1);
+          if (ok && it >= 2) ok = mbar_wait(bar(BAR_O_DONE + st), ((it - 2) >> 1) & 1);
           if (!ok) break;
           tc_fence_after();
 #pragma unroll
@@ -402,12 +409,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
 #pragma unroll
           for (int kk = 0; kk < kBN / 16; ++kk) {
-            const uint32_t pa = p_base + (kk >> 2) * kRegion + (kk & 3) * 32;
+            // P(jt) in S buffer jt&1: 16 keys per MMA = 8 TMEM columns
+            const uint32_t pa = tmem + (uint32_t)(sp * 128 + kk * 8);
             const uint32_t va = v_base + sp * L::kKVBytes + kk * 16 * 128;
-            tc_mma_f16(tmem_O, smem_desc_sw128(pa, 16, 1024), smem_desc_sw128(va, kRegion, 1024),
-                       kIdO, (jt > 0 || kk > 0) ? 1u : 0u);
+            tc_mma_f16_ts(tmem_O, pa, smem_desc_sw128(va, kRegion, 1024), kIdO,
+                          (jt > 0 || kk > 0) ? 1u : 0u);
           }
-          tc_commit(bar(BAR_O_DONE));
+          tc_commit(bar(BAR_O_DONE + sp));
           tc_commit(bar(BAR_V_EMPTY + sp));
         }
       }
@@ -451,6 +459,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     const uint32_t tmem_O = tmem + 256u;
     float m_run = NEG_INF, l_run = 0.f;  // m_run in raw score units
+    // PV products observed so far, in order (PV(j): barrier j & 1, phase j >> 1)
+    int o_seen = 0;
+    auto observe = [&](int upto) -> bool {
+      bool good = true;
+      while (good && o_seen < upto) {
+        good = mbar_wait(bar(BAR_O_DONE + (o_seen & 1)), (o_seen >> 1) & 1);
+        if (good) ++o_seen;
+      }
+      return good;
+    };
     // Every softmax warp runs the same number of iterations and meets the
     // named barrier in each one, also after a timed-out wait (then it only
     // skips the work), so no warp is ever left waiting at that barrier.
@@ -462,6 +480,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       float s[64];
       float mx = NEG_INF;
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_S_FULL + st), (it >> 1) & 1));
+      // S(it) began after PV(it-2) finished: observing PV(0..it-2) returns at once
+      if (ok) ok = __all_sync(0xffffffffu, observe(it - 1));
       if (ok) {
         tc_fence_after();
         const uint32_t ts = tmem + (uint32_t)(st * 128) + lane_off + half * 64;
@@ -487,7 +507,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       rm[half * kBM + r] = mx;
       softmax_bar();
       if (!ok) continue;
-      const float m_new = fmaxf(m_run, fmaxf(rm[r], rm[kBM + r]));
+      // The reference max only moves when the row max grows by more than 8
+      // (base 2): P = 2^(s - m_ref) stays below 2^8, exact enough in bf16 and
+      // far from fp32 overflow, and most tiles skip the rescale of O.  O, l
+      // and the partial rows all use the same reference.
+      const float m_max = fmaxf(m_run, fmaxf(rm[r], rm[kBM + r]));
+      const float m_new = (m_run == NEG_INF || (m_max - m_run) * sl2 > 8.f) ? m_max : m_run;
       const float m_use = (m_new == NEG_INF) ? 0.f : m_new;
       const float nb = -m_use * sl2;
       const float corr = ex2(fmaf(m_run, sl2, nb));
@@ -500,12 +525,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         rs1 += s[c + 1];
       }
       l_run = l_run * corr + (rs0 + rs1);
-      if (it > 0) {
-        // PV(it-1) must finish before O is rescaled and P is overwritten
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_O_DONE), (it - 1) & 1));
+      if (it > 0 && __any_sync(0xffffffffu, m_new > m_run)) {
+        // PV(it-1) must finish before O is rescaled
+        ok = __all_sync(0xffffffffu, observe(it));
         if (!ok) continue;
         tc_fence_after();
-        if (__any_sync(0xffffffffu, m_new > m_run)) {
+        {
 #pragma unroll
           for (int c = 0; c < DH / 32; ++c) {
             uint32_t o[32];
@@ -530,22 +555,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                          make_uint4(0u, 0u, 0u, 0u));
         }
       }
-      // this thread's 64 P columns -> region `half`, bf16, 128-byte swizzle
+      // this thread's 64 P values as bf16 pairs over its half of the S
+      // buffer: columns st*128 + half*32 .. +32 (both halves have read their
+      // S past the row-max barrier above)
+      {
+        uint32_t pw[32];
 #pragma unroll
-      for (int ch = 0; ch < 8; ++ch) {
-        const uint4 w = make_uint4(pack_bf16(s[ch * 8 + 0], s[ch * 8 + 1]),
-                                   pack_bf16(s[ch * 8 + 2], s[ch * 8 + 3]),
-                                   pack_bf16(s[ch * 8 + 4], s[ch * 8 + 5]),
-                                   pack_bf16(s[ch * 8 + 6], s[ch * 8 + 7]));
-        st_shared_v4(p_base + half * kRegion + r * 128 + ((ch ^ (r & 7)) << 4), w);
+        for (int w = 0; w < 32; ++w) pw[w] = pack_bf16(s[2 * w], s[2 * w + 1]);
+        tmem_st32(tmem + (uint32_t)(st * 128 + half * 32) + lane_off, pw);
+        tc_wait_st();
       }
-      fence_proxy_async_smem();
+      fence_proxy_async_smem();  // the zeroed V rows (generic stores) for the PV product
       tc_fence_before();
       mbar_arrive(bar(BAR_P_FULL));
       m_run = m_new;
     }
     if (ok && nt > 0) {
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_O_DONE), (nt - 1) & 1));
+      ok = __all_sync(0xffffffffu, observe(nt));
       if (ok) tc_fence_after();
     }
     // speculative K/V copies this split did not use land in the buffers the
