@@ -348,7 +348,8 @@ def grow_state():
                 new=[0], P=set(), lse_m={})
 
 
-def grow_step(state, a: int, W: int, m: int, small_logits, middle_logits, *, bf16: bool = False):
+def grow_step(state, a: int, W: int, m: int, small_logits, middle_logits, *, bf16: bool = False,
+              small_draft=None):
     """One drafting step k of Algorithm 2 on `state` (see grow_state), in place.
 
     The drafters' next-token logits under the prefix ending at node v are
@@ -365,6 +366,10 @@ def grow_step(state, a: int, W: int, m: int, small_logits, middle_logits, *, bf1
     v in F gets its m best middle-drafter tokens; then P = P u C.  Children
     are appended in frontier order, then child rank, never replacing an
     existing node.  Returns the frontier F.
+
+    small_draft, if given, replaces the small drafter's table: a callable
+    (state, v, m) -> (tokens, log-probabilities) giving v's m children (the
+    training-free n-gram drafter of the Appendix; oracle/ngram_oracle.py).
     """
     parent, token, edge, score = state["parent"], state["token"], state["edge"], state["score"]
     P, lse_m = state["P"], state["lse_m"]
@@ -386,6 +391,15 @@ def grow_step(state, a: int, W: int, m: int, small_logits, middle_logits, *, bf1
     F = sorted(C, key=lambda v: (-float(score[v]), v))[:W]
     made = []
     for v in F:
+        if a == 0 and small_draft is not None:
+            toks, lps = small_draft(state, v, m)
+            for y, lp in zip(toks, lps):
+                parent.append(v)
+                token.append(int(y))
+                edge.append(np.float32(lp))
+                score.append(np.float32(score[v] + np.float32(lp)))
+                made.append(len(parent) - 1)
+            continue
         x, lse = _row_log_softmax(table, v, bf16)
         order = np.lexsort((np.arange(len(x)), -x))[:m]
         for y in order:
