@@ -338,6 +338,84 @@ int treegraft_grow_step(int mode, const void* logits, int dtype, int V, int64_t 
                         size_t ws_bytes, void* stream);
 
 /*
+ * n-gram small drafter (Appendix, "n-gram small drafter"; the small drafter
+ * of Algorithm 2).  A training-free lookup: at prefill the target's top
+ * m_cache next-token candidates and their log-probabilities are cached at
+ * every prompt position, and an n-gram index is built over the prompt; at a
+ * small-drafter step the suffix of the prefix at tree node v is matched in
+ * the prompt with the longest n-gram that occurs (max_n tokens, then one
+ * fewer, ... down to one), at the n-gram's latest occurrence, and the
+ * candidates cached at the matched position become v's children, their
+ * cached log-probabilities the edge scores p(u).  With no match at any
+ * length the position of the prompt's most frequent token (ties to the
+ * lower token id; its latest occurrence) is used.
+ *
+ * Prompts are packed: `tokens` int32 [n_tokens], sequence b owns positions
+ * [seq_off[b], seq_off[b + 1]) (seq_off int32 [B + 1] on the device,
+ * seq_off[0] = 0, strictly increasing: every prompt non-empty,
+ * seq_off[B] = n_tokens).  Tree b of a draft or grow call belongs to prompt b.
+ * The prefix at node v is the committed text followed by the tokens of the
+ * non-root nodes on the path root -> v: the committed text's last max_n
+ * tokens are ctx[b * max_n + 0 .. ctx_len[b]) (int32 [B, max_n] and [B] on
+ * the device, oldest first; its last token is the root's, so token[root] is
+ * not read; 0 <= ctx_len[b] <= max_n).  Only the prompt is indexed (its
+ * positions are the ones with cached candidates); a match lies wholly
+ * inside one prompt.
+ *
+ * treegraft_ngram_index_bytes: bytes of the index for (B, n_tokens,
+ *   max_n); 0 for an invalid or unsupported shape.
+ * treegraft_ngram_build: build the index into `index` (caller-owned device
+ *   buffer, 16-byte aligned, no initial contents required; it keeps its own
+ *   copy of the tokens).  Four launches.  A malformed seq_off sets
+ *   TG_ERR_DEVICE_INDEX (the index is then unusable).
+ * treegraft_ngram_cache: the prefill cache from the prefill logits [rows,
+ *   ld] (row i = the target's next-token logits after packed position i, so
+ *   rows = n_tokens): cache_tok int32 [rows, m_cache] by (logit desc, token
+ *   asc), cache_lp fp32 [rows, m_cache] = fp32(logit - lse).  One
+ *   expand_topk launch.
+ * treegraft_ngram_draft: the drafter's expansion of arbitrary tree nodes:
+ *   rows int32 [R] (device) = b * cap + v; parent, token int32 [B * cap]
+ *   (tree b at rows [b * cap, (b + 1) * cap), local ids, parents before
+ *   children); outputs tok int32, logprob, score fp32 [R, m] with score =
+ *   fp32(parent_score[r] + logprob) for the first m <= m_cache cached
+ *   candidates; match_pos int32 [R] (position within its prompt) and
+ *   match_n int32 [R] (the order matched, 0 for the fallback) may be NULL.
+ *   One launch, one warp per row.
+ * treegraft_ngram_grow_step: one small-drafter step of Algorithm 2 with this
+ *   drafter on B trees of capacity cap (the tree layout, n, pool_lo, W, m
+ *   and frontier of treegraft_grow_step with mode 0): F = Top_W of the pool
+ *   [pool_lo, n) by (s desc, id asc), each node of F gets the first m
+ *   candidates of its lookup as children, appended at n, n + 1, ... in
+ *   frontier order then candidate rank, edge = the cached log-probability,
+ *   score = fp32(s(v) + edge).  One launch, one CTA per tree.
+ * Errors: TG_ERR_INVALID_ARG (null pointer, sizes, m > m_cache, a small
+ *   index buffer, capacity overflow), TG_ERR_UNSUPPORTED (max_n >
+ *   TG_NGRAM_MAX_N, n_tokens > TG_NGRAM_MAX_TOKENS, m_cache > TG_MAX_TOPK,
+ *   cap > TG_MAX_GROW_NODES), TG_ERR_CUDA.  On the device: a malformed tree
+ *   sets TG_ERR_DEVICE_TREE, a row outside [0, B * cap), a ctx_len outside
+ *   [0, max_n] or a prompt with no fallback position sets
+ *   TG_ERR_DEVICE_INDEX; the affected outputs are then undefined.
+ */
+#define TG_NGRAM_MAX_N 8
+#define TG_NGRAM_MAX_TOKENS (1 << 26)
+size_t treegraft_ngram_index_bytes(int B, int n_tokens, int max_n);
+int treegraft_ngram_build(const int32_t* tokens, const int32_t* seq_off, int B, int n_tokens,
+                          int max_n, void* index, size_t index_bytes, void* stream);
+int treegraft_ngram_cache(const void* logits, int dtype, int rows, int V, int64_t ld, int m_cache,
+                          int32_t* cache_tok, float* cache_lp, void* stream);
+int treegraft_ngram_draft(const void* index, size_t index_bytes, int B, int n_tokens, int max_n,
+                          const int32_t* cache_tok, const float* cache_lp, int m_cache,
+                          const int32_t* ctx, const int32_t* ctx_len, const int32_t* parent,
+                          const int32_t* token, int cap, const int32_t* rows, int R,
+                          const float* parent_score, int m, int32_t* tok, float* logprob,
+                          float* score, int32_t* match_pos, int32_t* match_n, void* stream);
+int treegraft_ngram_grow_step(const void* index, size_t index_bytes, int B, int n_tokens,
+                              int max_n, const int32_t* cache_tok, const float* cache_lp,
+                              int m_cache, const int32_t* ctx, const int32_t* ctx_len, int cap,
+                              int n, int pool_lo, int W, int m, int32_t* parent, int32_t* token,
+                              float* edge, float* score, int32_t* frontier, void* stream);
+
+/*
  * treegraft_last_device_status - synchronise `stream`, return the OR of the
  * device status bits raised since the last call on the current device
  * (TG_OK if none), and clear them.  Returns TG_ERR_CUDA if the

@@ -22,6 +22,7 @@ MAX_TREE_NODES = 256
 MAX_TOPK = 32
 MAX_PRUNE_NODES = 1024
 MAX_GROW_NODES = 1024
+NGRAM_MAX_N = 8
 
 _lib = None
 
@@ -57,11 +58,21 @@ _SIGNATURES = {
     "treegraft_grow_step": [_c_int, _c_vp, _c_int, _c_int, _c_i64, _c_int, _c_int, _c_int, _c_int,
                             _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp,
                             _c_size, _c_vp],
+    "treegraft_ngram_index_bytes": [_c_int, _c_int, _c_int],
+    "treegraft_ngram_build": [_c_vp, _c_vp, _c_int, _c_int, _c_int, _c_vp, _c_size, _c_vp],
+    "treegraft_ngram_cache": [_c_vp, _c_int, _c_int, _c_int, _c_i64, _c_int, _c_vp, _c_vp, _c_vp],
+    "treegraft_ngram_draft": [_c_vp, _c_size, _c_int, _c_int, _c_int, _c_vp, _c_vp, _c_int, _c_vp,
+                              _c_vp, _c_vp, _c_vp, _c_int, _c_vp, _c_int, _c_vp, _c_int, _c_vp,
+                              _c_vp, _c_vp, _c_vp, _c_vp, _c_vp],
+    "treegraft_ngram_grow_step": [_c_vp, _c_size, _c_int, _c_int, _c_int, _c_vp, _c_vp, _c_int,
+                                  _c_vp, _c_vp, _c_int, _c_int, _c_int, _c_int, _c_int, _c_vp,
+                                  _c_vp, _c_vp, _c_vp, _c_vp, _c_vp],
     "treegraft_last_device_status": [_c_vp],
     "treegraft_status_string": [_c_int],
 }
 _RESTYPES = {"treegraft_accept_workspace_size": _c_size,
              "treegraft_grow_workspace_size": _c_size,
+             "treegraft_ngram_index_bytes": _c_size,
              "treegraft_tree_attn_workspace_size": _c_size,
              "treegraft_status_string": ctypes.c_char_p}
 
@@ -348,4 +359,113 @@ def grow_step(mode, logits, W, m, parent, token, edge, score, n, pool_lo, *, lse
                                    _ptr(edge), _ptr(score), _ptr(lse_mid), _ptr(frontier), _ptr(ws),
                                    ws.numel(), _stream(stream))
     _check("treegraft_grow_step", st)
+    return frontier
+
+
+class NgramIndex:
+    """The n-gram small drafter's prompt index (a device buffer built by
+    ngram_build) with the shape it was built for."""
+
+    def __init__(self, buf, B, n_tokens, max_n):
+        self.buf, self.B, self.n_tokens, self.max_n = buf, int(B), int(n_tokens), int(max_n)
+
+
+def ngram_index_bytes(B, n_tokens, max_n) -> int:
+    return int(lib().treegraft_ngram_index_bytes(int(B), int(n_tokens), int(max_n)))
+
+
+def ngram_build(tokens, seq_off, max_n, *, index=None, stream=None):
+    """Build the n-gram index over packed prompts: tokens int32 [n_tokens],
+    seq_off int32 [B + 1] (prompt b = tokens[seq_off[b]:seq_off[b + 1]])."""
+    _need(tokens, torch.int32, "tokens")
+    _need(seq_off, torch.int32, "seq_off")
+    B, n_tokens = seq_off.numel() - 1, tokens.numel()
+    nbytes = ngram_index_bytes(B, n_tokens, max_n)
+    if nbytes == 0:
+        raise ValueError("ngram index: unsupported sizes")
+    buf = index.buf if index is not None else torch.empty(nbytes, dtype=torch.uint8,
+                                                          device=tokens.device)
+    st = lib().treegraft_ngram_build(_ptr(tokens), _ptr(seq_off), B, n_tokens, int(max_n),
+                                     _ptr(buf), buf.numel(), _stream(stream))
+    _check("treegraft_ngram_build", st)
+    return NgramIndex(buf, B, n_tokens, max_n)
+
+
+def ngram_cache(logits, m_cache, *, cache_tok=None, cache_lp=None, V=None, stream=None):
+    """Prefill cache: the top-m_cache tokens (int32) and log-probabilities
+    (fp32) of every row of the prefill logits [n_tokens, ld]."""
+    if logits.dim() != 2 or logits.stride(1) != 1 or not logits.is_cuda:
+        raise ValueError("logits must be a 2-D CUDA tensor with unit column stride")
+    rows = logits.shape[0]
+    V = logits.shape[1] if V is None else int(V)
+    if cache_tok is None:
+        cache_tok = torch.empty(rows, int(m_cache), dtype=torch.int32, device=logits.device)
+    if cache_lp is None:
+        cache_lp = torch.empty(rows, int(m_cache), dtype=torch.float32, device=logits.device)
+    _need(cache_tok, torch.int32, "cache_tok")
+    _need(cache_lp, torch.float32, "cache_lp")
+    st = lib().treegraft_ngram_cache(_ptr(logits), _logit_dtype(logits), rows, V, logits.stride(0),
+                                     int(m_cache), _ptr(cache_tok), _ptr(cache_lp), _stream(stream))
+    _check("treegraft_ngram_cache", st)
+    return cache_tok, cache_lp
+
+
+def _ngram_common(index, cache_tok, cache_lp, ctx, ctx_len):
+    _need(cache_tok, torch.int32, "cache_tok")
+    _need(cache_lp, torch.float32, "cache_lp")
+    _need(ctx, torch.int32, "ctx")
+    _need(ctx_len, torch.int32, "ctx_len")
+    if (cache_tok.dim() != 2 or cache_tok.shape != cache_lp.shape
+            or cache_tok.shape[0] != index.n_tokens):
+        raise ValueError("cache_tok / cache_lp must be [n_tokens, m_cache]")
+    if tuple(ctx.shape) != (index.B, index.max_n):
+        raise ValueError("ctx must be [B, max_n]")
+    return (_ptr(index.buf), index.buf.numel(), index.B, index.n_tokens, index.max_n,
+            _ptr(cache_tok), _ptr(cache_lp), cache_tok.shape[1], _ptr(ctx), _ptr(ctx_len))
+
+
+def ngram_draft(index, cache_tok, cache_lp, ctx, ctx_len, parent, token, rows, parent_score, m,
+                *, with_match=False, stream=None):
+    """The n-gram drafter's expansion of tree nodes rows int32 [R] (= b * cap
+    + v) on trees parent / token int32 [B, cap]: tok int32, logprob, score
+    fp32 [R, m] (and the matched prompt position and order if with_match)."""
+    for t, nm in ((parent, "parent"), (token, "token"), (rows, "rows")):
+        _need(t, torch.int32, nm)
+    _need(parent_score, torch.float32, "parent_score")
+    if parent.dim() != 2:
+        raise ValueError("tree arrays must be [B, cap]")
+    R, dev = rows.numel(), rows.device
+    tok = torch.empty(R, int(m), dtype=torch.int32, device=dev)
+    lp = torch.empty(R, int(m), dtype=torch.float32, device=dev)
+    sc = torch.empty(R, int(m), dtype=torch.float32, device=dev)
+    pos = torch.empty(R, dtype=torch.int32, device=dev) if with_match else None
+    nn = torch.empty(R, dtype=torch.int32, device=dev) if with_match else None
+    st = lib().treegraft_ngram_draft(*_ngram_common(index, cache_tok, cache_lp, ctx, ctx_len),
+                                     _ptr(parent), _ptr(token), parent.shape[1], _ptr(rows), R,
+                                     _ptr(parent_score), int(m), _ptr(tok), _ptr(lp), _ptr(sc),
+                                     _ptr(pos), _ptr(nn), _stream(stream))
+    _check("treegraft_ngram_draft", st)
+    return (tok, lp, sc, pos, nn) if with_match else (tok, lp, sc)
+
+
+def ngram_grow_step(index, cache_tok, cache_lp, ctx, ctx_len, W, m, parent, token, edge, score, n,
+                    pool_lo, *, frontier=None, stream=None):
+    """One small-drafter step of Algorithm 2 with the n-gram drafter on trees
+    parent / token int32, edge / score fp32 [B, cap] (updated in place).
+    Returns the frontier int32 [B, W]."""
+    for t, nm in ((parent, "parent"), (token, "token")):
+        _need(t, torch.int32, nm)
+    for t, nm in ((edge, "edge"), (score, "score")):
+        _need(t, torch.float32, nm)
+    if parent.dim() != 2:
+        raise ValueError("tree arrays must be [B, cap]")
+    B, cap = parent.shape
+    if frontier is None:
+        frontier = torch.empty(B, int(W), dtype=torch.int32, device=parent.device)
+    _need(frontier, torch.int32, "frontier")
+    st = lib().treegraft_ngram_grow_step(*_ngram_common(index, cache_tok, cache_lp, ctx, ctx_len),
+                                         cap, int(n), int(pool_lo), int(W), int(m), _ptr(parent),
+                                         _ptr(token), _ptr(edge), _ptr(score), _ptr(frontier),
+                                         _stream(stream))
+    _check("treegraft_ngram_grow_step", st)
     return frontier

@@ -91,6 +91,32 @@ int device_sm_count() {
 
 int* status_word_ptr() { return status_ptr(); }
 
+namespace {
+bool ngram_shape_ok(int B, int n_tokens, int max_n) {
+  return B >= 1 && n_tokens >= B && max_n >= 1 && max_n <= TG_NGRAM_MAX_N;
+}
+bool ngram_shape_supported(int n_tokens) { return n_tokens <= TG_NGRAM_MAX_TOKENS; }
+
+// index, cache and context arguments shared by draft and grow
+int ngram_common(NgramArgs& a, const void* index, size_t index_bytes, int B, int n_tokens,
+                 int max_n, const int32_t* cache_tok, const float* cache_lp, int m_cache,
+                 const int32_t* ctx, const int32_t* ctx_len, int m) {
+  if (!index || !cache_tok || !cache_lp || !ctx || !ctx_len) return TG_ERR_INVALID_ARG;
+  if (!ngram_shape_ok(B, n_tokens, max_n) || m < 1 || m_cache < m) return TG_ERR_INVALID_ARG;
+  if (!ngram_shape_supported(n_tokens) || m_cache > TG_MAX_TOPK) return TG_ERR_UNSUPPORTED;
+  if (index_bytes < ngram_layout(B, n_tokens, max_n).total || !aligned16(index))
+    return TG_ERR_INVALID_ARG;
+  ngram_carve(a, const_cast<void*>(index), B, n_tokens, max_n);
+  a.cache_tok = cache_tok;
+  a.cache_lp = cache_lp;
+  a.m_cache = m_cache;
+  a.ctx = ctx;
+  a.ctx_len = ctx_len;
+  a.m = m;
+  return TG_OK;
+}
+}  // namespace
+
 }  // namespace tg
 
 using namespace tg;
@@ -358,6 +384,122 @@ int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld, co
   a.tickets = static_cast<int32_t*>(ws) + n_total;
   a.status = st;
   return launch_accept(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK : TG_ERR_CUDA;
+}
+
+
+size_t treegraft_ngram_index_bytes(int B, int n_tokens, int max_n) {
+  if (!ngram_shape_ok(B, n_tokens, max_n) || !ngram_shape_supported(n_tokens)) return 0;
+  return ngram_layout(B, n_tokens, max_n).total;
+}
+
+int treegraft_ngram_build(const int32_t* tokens, const int32_t* seq_off, int B, int n_tokens,
+                          int max_n, void* index, size_t index_bytes, void* stream) {
+  if (!tokens || !seq_off || !index) return TG_ERR_INVALID_ARG;
+  if (!ngram_shape_ok(B, n_tokens, max_n)) return TG_ERR_INVALID_ARG;
+  if (!ngram_shape_supported(n_tokens)) return TG_ERR_UNSUPPORTED;
+  if (index_bytes < ngram_layout(B, n_tokens, max_n).total || !aligned16(index))
+    return TG_ERR_INVALID_ARG;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  NgramArgs a = {};
+  ngram_carve(a, index, B, n_tokens, max_n);
+  a.src_tok = tokens;
+  a.src_seq = seq_off;
+  a.status = st;
+  return launch_ngram_build(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK
+                                                                              : TG_ERR_CUDA;
+}
+
+int treegraft_ngram_cache(const void* logits, int dtype, int rows, int V, int64_t ld, int m_cache,
+                          int32_t* cache_tok, float* cache_lp, void* stream) {
+  if (rows == 0) return TG_OK;
+  if (!logits || !cache_tok || !cache_lp) return TG_ERR_INVALID_ARG;
+  if (dtype != TG_BF16 && dtype != TG_F32) return TG_ERR_INVALID_ARG;
+  if (rows < 0 || V < 1 || ld < V || m_cache < 1 || m_cache > V) return TG_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(logits) & (dtype == TG_BF16 ? 1 : 3)) != 0)
+    return TG_ERR_INVALID_ARG;
+  if (m_cache > TG_MAX_TOPK || V > (dtype == TG_BF16 ? 262144 : 131072)) return TG_ERR_UNSUPPORTED;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  TopkArgs a = {};
+  a.logits = logits;
+  a.is_bf16 = dtype == TG_BF16;
+  a.logit_rows = rows;
+  a.V = V;
+  a.ld = ld;
+  a.rows = rows;
+  a.row_idx = nullptr;
+  a.parent_score = nullptr;  // log-probabilities only
+  a.k = m_cache;
+  a.tok = cache_tok;
+  a.logprob = cache_lp;
+  a.score = nullptr;
+  a.lse_out = nullptr;
+  a.status = st;
+  return launch_expand_topk(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK
+                                                                               : TG_ERR_CUDA;
+}
+
+int treegraft_ngram_draft(const void* index, size_t index_bytes, int B, int n_tokens, int max_n,
+                          const int32_t* cache_tok, const float* cache_lp, int m_cache,
+                          const int32_t* ctx, const int32_t* ctx_len, const int32_t* parent,
+                          const int32_t* token, int cap, const int32_t* rows, int R,
+                          const float* parent_score, int m, int32_t* tok, float* logprob,
+                          float* score, int32_t* match_pos, int32_t* match_n, void* stream) {
+  if (R == 0) return TG_OK;
+  if (R < 0 || cap < 1 || !parent || !token || !rows || !parent_score || !tok || !logprob || !score)
+    return TG_ERR_INVALID_ARG;
+  if ((long long)B * cap > (1ll << 30)) return TG_ERR_UNSUPPORTED;
+  NgramArgs a = {};
+  const int e = ngram_common(a, index, index_bytes, B, n_tokens, max_n, cache_tok, cache_lp,
+                             m_cache, ctx, ctx_len, m);
+  if (e != TG_OK) return e;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  a.parent = const_cast<int32_t*>(parent);
+  a.token = const_cast<int32_t*>(token);
+  a.cap = cap;
+  a.rows = rows;
+  a.R = R;
+  a.parent_score = parent_score;
+  a.out_tok = tok;
+  a.out_lp = logprob;
+  a.out_score = score;
+  a.match_pos = match_pos;
+  a.match_n = match_n;
+  a.status = st;
+  return launch_ngram_draft(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK
+                                                                              : TG_ERR_CUDA;
+}
+
+int treegraft_ngram_grow_step(const void* index, size_t index_bytes, int B, int n_tokens,
+                              int max_n, const int32_t* cache_tok, const float* cache_lp,
+                              int m_cache, const int32_t* ctx, const int32_t* ctx_len, int cap,
+                              int n, int pool_lo, int W, int m, int32_t* parent, int32_t* token,
+                              float* edge, float* score, int32_t* frontier, void* stream) {
+  if (!parent || !token || !edge || !score || !frontier) return TG_ERR_INVALID_ARG;
+  if (cap < 1 || n < 1 || n > cap || pool_lo < 0 || pool_lo >= n || W < 1) return TG_ERR_INVALID_ARG;
+  if ((long long)n + (long long)std::min(W, n - pool_lo) * m > (long long)cap)
+    return TG_ERR_INVALID_ARG;  // the children would not fit the tree's capacity
+  if (cap > TG_MAX_GROW_NODES || (long long)B * cap > (1ll << 30)) return TG_ERR_UNSUPPORTED;
+  NgramArgs a = {};
+  const int e = ngram_common(a, index, index_bytes, B, n_tokens, max_n, cache_tok, cache_lp,
+                             m_cache, ctx, ctx_len, m);
+  if (e != TG_OK) return e;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  a.parent = parent;
+  a.token = token;
+  a.cap = cap;
+  a.n = n;
+  a.pool_lo = pool_lo;
+  a.W = W;
+  a.edge = edge;
+  a.score = score;
+  a.frontier = frontier;
+  a.status = st;
+  return launch_ngram_grow(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK
+                                                                             : TG_ERR_CUDA;
 }
 
 int treegraft_last_device_status(void* stream) {

@@ -131,6 +131,55 @@ size_t grow_ws_bytes(int B, int cap, int m);
 void grow_ws_carve(GrowArgs& a, void* ws, int B, int cap, int m);
 cudaError_t launch_grow_step(const GrowArgs& a, cudaStream_t s);
 
+// n-gram small drafter: the index lives in one caller buffer (ngram_layout)
+struct NgramLayout {
+  size_t tok, seq, tab, cnt, fbk, fbp, total;  // byte offsets, 256-aligned
+  int T;                                       // slots per order
+};
+struct NgramArgs {
+  // index (ngram_carve)
+  int32_t* tok;              // [n_tokens] packed prompt tokens
+  int32_t* seq;              // [B + 1] sequence offsets
+  int32_t* tab;              // [max_n][T] latest position per n-gram, -1 empty
+  int32_t* cnt;              // [T] occurrences per order-1 slot
+  unsigned long long* fbk;   // [B] (count, -token) of the most frequent token
+  int32_t* fbp;              // [B] its latest position (-1: none)
+  int T, B, n_tokens, max_n;
+  // build
+  const int32_t* src_tok;
+  const int32_t* src_seq;
+  // lookup
+  const int32_t* cache_tok;  // [n_tokens, m_cache]
+  const float* cache_lp;
+  int m_cache;
+  const int32_t* ctx;        // [B, max_n] committed tail, oldest first
+  const int32_t* ctx_len;    // [B]
+  int32_t* parent;           // [B * cap] trees
+  int32_t* token;
+  int cap;
+  // draft
+  const int32_t* rows;       // [R] b * cap + v
+  int R;
+  const float* parent_score;
+  int m;
+  int32_t* out_tok;
+  float* out_lp;
+  float* out_score;
+  int32_t* match_pos;
+  int32_t* match_n;
+  // grow
+  int n, pool_lo, W;
+  float* edge;
+  float* score;
+  int32_t* frontier;
+  int* status;
+};
+NgramLayout ngram_layout(int B, int n_tokens, int max_n);
+void ngram_carve(NgramArgs& a, void* index, int B, int n_tokens, int max_n);
+cudaError_t launch_ngram_build(const NgramArgs& a, cudaStream_t s);
+cudaError_t launch_ngram_draft(const NgramArgs& a, cudaStream_t s);
+cudaError_t launch_ngram_grow(const NgramArgs& a, cudaStream_t s);
+
 int device_sm_count();
 // device address of the per-device status word (nullptr on failure)
 int* status_word_ptr();

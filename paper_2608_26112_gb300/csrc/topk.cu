@@ -237,7 +237,7 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   // the leader's threads fetch the parent's path score now, while the
   // logits are in flight (one broadcast request per warp)
   float parent_score = 0.f;
-  if (crank == 0) parent_score = __ldg(a.parent_score + row);
+  if (crank == 0 && a.parent_score) parent_score = __ldg(a.parent_score + row);
   const int per = ((V + C - 1) / C + VW - 1) / VW * VW;
   const int c0 = min(V, crank * per);
   const int c1 = min(V, c0 + per);
@@ -296,7 +296,7 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
       const size_t o = (size_t)row * k + rank;
       a.tok[o] = (int32_t)key_index(key);
       a.logprob[o] = lp;
-      a.score[o] = __fadd_rn(parent_score, lp);
+      if (a.score) a.score[o] = __fadd_rn(parent_score, lp);
       if (rank == 0 && a.lse_out) a.lse_out[row] = lse;
     }
   }
@@ -319,10 +319,10 @@ cudaError_t launch_topk_t(const TopkArgs& a, int C, cudaStream_t s) {
       b.logits = static_cast<const char*>(a.logits) + (size_t)r0 * (size_t)a.ld * (a.is_bf16 ? 2 : 4);
       b.logit_rows = a.logit_rows - r0;
     }
-    b.parent_score += r0;
+    if (b.parent_score) b.parent_score += r0;
     b.tok += (size_t)r0 * a.k;
     b.logprob += (size_t)r0 * a.k;
-    b.score += (size_t)r0 * a.k;
+    if (b.score) b.score += (size_t)r0 * a.k;
     if (b.lse_out) b.lse_out += r0;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(C, nr, 1);

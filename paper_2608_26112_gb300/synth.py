@@ -170,6 +170,46 @@ def plant_child_bump(rng, logits: np.ndarray, parent: np.ndarray, token: np.ndar
             logits[row_of_node[v], token[c]] += np.float32(bump)
 
 
+# --------------------------------------------------------------------------
+# prompts for the n-gram small drafter
+# --------------------------------------------------------------------------
+
+def prompt_stream(rng, L: int, V: int, *, copy_prob: float = 0.1, seg: tuple = (2, 12),
+                  zipf_a: float = 1.1, active: int = 4096) -> np.ndarray:
+    """A synthetic prompt of L tokens (int32) with the reuse that makes an
+    n-gram drafter useful: each new piece is, with probability copy_prob, a
+    copy of an earlier segment of length uniform in [seg[0], seg[1]],
+    otherwise one token drawn from a Zipf(zipf_a) law over `active` tokens
+    of a random permutation of the vocabulary."""
+    active = min(active, V)
+    vocab = rng.permutation(V)[:active]
+    w = 1.0 / np.arange(1, active + 1) ** zipf_a
+    draws = vocab[rng.choice(active, size=L, p=w / w.sum())]
+    out = np.empty(L, np.int64)
+    i = 0
+    while i < L:
+        if i >= seg[0] and rng.random() < copy_prob:
+            ln = int(rng.integers(seg[0], seg[1] + 1))
+            st = int(rng.integers(0, i - seg[0] + 1))
+            ln = min(ln, L - i, i - st)
+            out[i:i + ln] = out[st:st + ln]
+            i += ln
+        else:
+            out[i] = draws[i]
+            i += 1
+    return out.astype(np.int32)
+
+
+def plant_next_token_bump(rng, logits: np.ndarray, prompt: np.ndarray, prob: float = 0.7,
+                          bump: float = 8.0) -> None:
+    """Prefill logits that often predict the text: for each position j but
+    the last, with probability `prob` add `bump` to row j's logit of the
+    prompt's next token prompt[j + 1] (in place, float32 [L, V])."""
+    for j in range(len(prompt) - 1):
+        if rng.random() < prob:
+            logits[j, prompt[j + 1]] += np.float32(bump)
+
+
 def kv_cache(rng, B: int, Hkv: int, S_max: int, D: int, valid: list[int],
              tail: str = "zero") -> np.ndarray:
     """bf16 bits [B, Hkv, S_max, D] drawn N(0,1) over the valid slots of each

@@ -167,3 +167,35 @@ def test_grow_step_rejects_bad_args_on_host(lib):
     assert call(cap=2000, n=11) == 2            # beyond TG_MAX_GROW_NODES
     assert call(m=33, V=100, cap=1024) == 2     # beyond TG_MAX_TOPK
     assert call(logits=ctypes.c_void_p(0x1001)) == 1  # misaligned bf16 elements
+
+
+def test_ngram_rejects_bad_args_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    need = lib.treegraft_ngram_index_bytes(2, 100, 4)
+    # T = 256 slots per order (>= 2 * 100): tokens, offsets, 4 tables, counts, fallbacks
+    assert need == 512 + 256 + 4 * 256 * 4 + 256 * 4 + 256 + 256
+    assert lib.treegraft_ngram_index_bytes(2, 100, 9) == 0          # max_n > TG_NGRAM_MAX_N
+    assert lib.treegraft_ngram_index_bytes(3, 2, 4) == 0            # an empty prompt
+    assert lib.treegraft_ngram_index_bytes(1, (1 << 26) + 1, 4) == 0
+    assert lib.treegraft_ngram_build(fake, fake, 2, 100, 4, fake, need - 1, NULL) == 1
+    assert lib.treegraft_ngram_build(NULL, fake, 2, 100, 4, fake, need, NULL) == 1
+    assert lib.treegraft_ngram_build(fake, fake, 2, 100, 9, fake, 1 << 20, NULL) == 1
+    assert lib.treegraft_ngram_cache(fake, 0, 10, 100, 100, 33, fake, fake, NULL) == 2
+    assert lib.treegraft_ngram_cache(fake, 0, 10, 100, 99, 4, fake, fake, NULL) == 1
+
+    def draft(m=4, m_cache=8, nbytes=need, R=5, index=fake):
+        return lib.treegraft_ngram_draft(index, nbytes, 2, 100, 4, fake, fake, m_cache, fake, fake,
+                                         fake, fake, 16, fake, R, fake, m, fake, fake, fake, NULL,
+                                         NULL, NULL)
+    assert draft(R=0) == 0
+    assert draft(m=9) == 1                   # m > m_cache
+    assert draft(m_cache=33, m=4) == 2
+    assert draft(nbytes=need - 256) == 1
+    assert draft(index=NULL) == 1
+
+    def grow(cap=64, n=5, pool_lo=1, W=4, m=4):
+        return lib.treegraft_ngram_grow_step(fake, need, 2, 100, 4, fake, fake, 8, fake, fake, cap,
+                                             n, pool_lo, W, m, fake, fake, fake, fake, fake, NULL)
+    assert grow(cap=20) == 1                 # 5 + 4 * 4 children do not fit
+    assert grow(pool_lo=5) == 1
+    assert grow(cap=2048, n=5) == 2          # beyond TG_MAX_GROW_NODES
