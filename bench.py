@@ -395,6 +395,107 @@ def grow_timing(seed, dev, stream, reps, n_sets=3):
             "note": "Algorithm 2 grow loop; bytes = drafter-table rows scanned x V x 2"}
 
 
+NGRAM_PROMPT, NGRAM_MAX_N, NGRAM_M_CACHE = 2048, 4, 10
+
+
+def ngram_timing(seed, dev, stream, reps, n_sets=3):
+    """The n-gram small drafter (the paper's training-free small drafter)
+    timed beside the step: its prefill work on a 2048-token prompt (the top-10
+    cache over 2048 rows of seeded N(0, 3^2) bf16 prefill logits, 128256
+    tokens, next-token bump; the order-1..4 index build), then Algorithm 2
+    with its small steps: the schedule [1, 0, 1, 0, 1] with W = m = 10 (the
+    middle steps on drafter tables as in the grow loop) and the all-small
+    schedule [0, 0, 0, 0, 0] (Algorithm 1 with this drafter), one tree from
+    the prompt's last token, n_sets rotating trees and tables."""
+    import numpy as np
+    import torch
+    import paper_2608_26112_gb300 as tg
+    from paper_2608_26112_gb300 import synth
+
+    W = m = 10
+    V, L, max_n, mc = 128256, NGRAM_PROMPT, NGRAM_MAX_N, NGRAM_M_CACHE
+    rng = synth.make_rng(40_000 + seed)
+    prompt = synth.prompt_stream(rng, L, V)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(40_000 + seed)
+    lg = torch.randn(L, V, generator=gen, device=dev, dtype=torch.float32).mul_(3.0)
+    nxt = torch.from_numpy(prompt[1:].astype(np.int64)).to(dev)
+    hit = torch.from_numpy(rng.random(L - 1) < 0.7).to(dev)
+    lg[torch.arange(L - 1, device=dev)[hit], nxt[hit]] += 8.0
+    lg = lg.to(torch.bfloat16)
+    toks = torch.from_numpy(prompt).to(dev)
+    seq = torch.tensor([0, L], dtype=torch.int32, device=dev)
+    ctok = torch.empty(L, mc, dtype=torch.int32, device=dev)
+    clp = torch.empty(L, mc, dtype=torch.float32, device=dev)
+    with torch.cuda.stream(stream):
+        index = tg.ngram_build(toks, seq, max_n, stream=stream)
+        tg.ngram_cache(lg, mc, cache_tok=ctok, cache_lp=clp, stream=stream)
+    stream.synchronize()
+    g_cache = capture(lambda: tg.ngram_cache(lg, mc, cache_tok=ctok, cache_lp=clp, stream=stream),
+                      stream)
+    g_build = capture(lambda: tg.ngram_build(toks, seq, max_n, index=index, stream=stream), stream)
+    g_cache.replay()
+    g_build.replay()
+    t_cache = time_graph(g_cache, max(5, reps // 20), stream) / max(5, reps // 20)
+    t_build = time_graph(g_build, max(5, reps // 10), stream) / max(5, reps // 10)
+    ctx = torch.from_numpy(prompt[-max_n:].reshape(1, max_n).astype(np.int32)).to(dev)
+    clen = torch.tensor([max_n], dtype=torch.int32, device=dev)
+
+    def plan(schedule):
+        sizes, n, new_lo, n_vis = [], 1, 0, 0
+        for a in schedule:
+            pool_lo = new_lo if a == 0 else n_vis
+            sizes.append((a, n, pool_lo))
+            if a == 1:
+                n_vis = n
+            new_lo, n = n, n + min(W, n - pool_lo) * m
+        return sizes, n
+
+    out = {"prompt_tokens": L, "max_n": max_n, "m_cache": mc, "vocab": V,
+           "cache_us": t_cache * 1e6, "cache_bytes": L * V * 2,
+           "cache_GBps": L * V * 2 / t_cache / 1e9, "build_us": t_build * 1e6,
+           "build_launches": 4, "in_step": False}
+    for label, schedule in (("grow_mixed", GROW_SCHEDULE), ("grow_small", [0] * 5)):
+        sizes, cap = plan(schedule)
+        sets = []
+        for r in range(n_sets):
+            rr = synth.make_rng(41_000 + seed + r)
+            mid = None
+            if 1 in schedule:
+                mid = torch.from_numpy(synth.f32_to_bf16_bits(synth.normal_f32(rr, (cap, V), 3.0))
+                                       .view(np.int16)).to(dev).view(torch.bfloat16)
+            sets.append((mid, dict(
+                parent=torch.full((1, cap), -1, dtype=torch.int32, device=dev),
+                token=torch.zeros(1, cap, dtype=torch.int32, device=dev),
+                edge=torch.zeros(1, cap, dtype=torch.float32, device=dev),
+                score=torch.zeros(1, cap, dtype=torch.float32, device=dev),
+                lse=torch.zeros(1, cap, dtype=torch.float32, device=dev),
+                fr=torch.empty(1, W, dtype=torch.int32, device=dev),
+                ws=tg.grow_workspace(1, cap, m, dev))))
+
+        def loop(mid, t, sizes=sizes):
+            for a, n_, lo in sizes:
+                if a == 1:
+                    tg.grow_step(1, mid, W, m, t["parent"], t["token"], t["edge"], t["score"], n_,
+                                 lo, lse_mid=t["lse"], frontier=t["fr"], ws=t["ws"], stream=stream)
+                else:
+                    tg.ngram_grow_step(index, ctok, clp, ctx, clen, W, m, t["parent"], t["token"],
+                                       t["edge"], t["score"], n_, lo, frontier=t["fr"],
+                                       stream=stream)
+
+        with torch.cuda.stream(stream):
+            for mid, t in sets:
+                loop(mid, t)
+        stream.synchronize()
+        g = capture(lambda: [loop(mid, t) for mid, t in sets], stream)
+        g.replay()
+        loops = max(5, reps // 10)
+        t = time_graph(g, loops, stream) / (loops * n_sets)
+        out[label] = {"schedule": schedule, "W": W, "m": m, "nodes_out": cap, "us": t * 1e6,
+                      "launches": sum(3 if a == 1 else 1 for a in schedule)}
+    return out
+
+
 # --------------------------------------------------------------------------- clocks
 
 class ClockSampler:
@@ -663,6 +764,7 @@ def ours_arm(args):
             kt[name] = time_graph(g, kreps, stream) / (kreps * R)
         prune = prune_timing(R, rank_seed(args.seed, rank), dev, stream, kreps)
         grow = grow_timing(rank_seed(args.seed, rank), dev, stream, kreps)
+        ngram = ngram_timing(rank_seed(args.seed, rank), dev, stream, kreps)
         extra = {nm: config_timing(nm, rank_seed(args.seed, rank), dev, stream)
                  for nm in EXTRA_CONFIGS}
     assert tg.last_device_status(stream) == 0
@@ -681,6 +783,7 @@ def ours_arm(args):
             kernels[name]["TFLOPs"] = f / kt[name] / 1e12
     kernels["global_prune"] = prune
     kernels["grow_loop"] = grow
+    kernels["ngram_drafter"] = ngram
     dom = max(KERNELS, key=lambda n: kt[n])
     b, f = costs[dom]
     achieved = b / kt[dom] / 1e9
