@@ -338,6 +338,42 @@ int treegraft_grow_step(int mode, const void* logits, int dtype, int V, int64_t 
                         size_t ws_bytes, void* stream);
 
 /*
+ * treegraft_accept_sample - verification at temperature T > 0: the tree
+ * rejection-sampling rule behind the distribution preservation of Sec. 3.2
+ * (Algorithms 1 and 2, verification step), for children that are
+ * deterministic proposals.  At node v (from the root) with p =
+ * softmax(target_logits[v] / T) and the residual r = p, v's children are
+ * visited in ascending node id; child c with token x is accepted iff
+ * u[c, 0] * sum(r) < r(x) (r holding p minus the tokens of the children
+ * rejected before c, so a child repeating an earlier sibling's token is
+ * never accepted); the walk moves to the first accepted child.  At the node
+ * a* where every child is rejected (or a leaf) the bonus token is drawn from
+ * r / sum(r) by inversion: the first token t whose cumulative residual mass
+ * exceeds u[a*, 1] * sum(r).  Each emitted token then follows p exactly.
+ *
+ * Trees, target_logits, path, accept_len and path_cap are as in
+ * treegraft_accept.  u: fp32 [n_total, 2] uniforms in [0, 1) on the
+ * device, drawn by the caller (u[c, 0] decides child c, u[v, 1] the bonus
+ * draw at v).  temperature > 0 (fp32 must be able to hold log2(e) / T).
+ * ws: treegraft_accept_sample_workspace_size(B, n_total) bytes, 16-byte
+ * aligned, ZEROED before its first use (per-tree tickets, reset by every
+ * call).  Two launches: per node row the (max, sum) and every child's
+ * decision, and the walk in the CTA that finishes a tree's rows; then row
+ * a* per tree for the bonus draw.  The comparisons are taken in fp32, so a
+ * draw within a few ulps of a threshold may fall either way.
+ * Errors: TG_ERR_INVALID_ARG, TG_ERR_UNSUPPORTED (V too large, B > 65535,
+ * T too small), TG_ERR_CUDA; a malformed tree sets TG_ERR_DEVICE_TREE and a
+ * token outside [0, V) or a path longer than path_cap TG_ERR_DEVICE_INDEX
+ * (that tree's outputs are then undefined).
+ */
+size_t treegraft_accept_sample_workspace_size(int B, int n_total);
+int treegraft_accept_sample(const void* target_logits, int dtype, int V, int64_t ld,
+                            float temperature, const int32_t* token, const int32_t* parent,
+                            const int32_t* node_off, int B, int max_nodes, int n_total,
+                            const float* u, int path_cap, int32_t* path, int32_t* accept_len,
+                            int32_t* bonus, void* ws, size_t ws_bytes, void* stream);
+
+/*
  * n-gram small drafter (Appendix, "n-gram small drafter"; the small drafter
  * of Algorithm 2).  A training-free lookup: at prefill the target's top
  * m_cache next-token candidates and their log-probabilities are cached at

@@ -58,6 +58,10 @@ _SIGNATURES = {
     "treegraft_grow_step": [_c_int, _c_vp, _c_int, _c_int, _c_i64, _c_int, _c_int, _c_int, _c_int,
                             _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp,
                             _c_size, _c_vp],
+    "treegraft_accept_sample_workspace_size": [_c_int, _c_int],
+    "treegraft_accept_sample": [_c_vp, _c_int, _c_int, _c_i64, _c_f32, _c_vp, _c_vp, _c_vp, _c_int,
+                                _c_int, _c_int, _c_vp, _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_size,
+                                _c_vp],
     "treegraft_ngram_index_bytes": [_c_int, _c_int, _c_int],
     "treegraft_ngram_build": [_c_vp, _c_vp, _c_int, _c_int, _c_int, _c_vp, _c_size, _c_vp],
     "treegraft_ngram_cache": [_c_vp, _c_int, _c_int, _c_int, _c_i64, _c_int, _c_vp, _c_vp, _c_vp],
@@ -73,6 +77,7 @@ _SIGNATURES = {
 _RESTYPES = {"treegraft_accept_workspace_size": _c_size,
              "treegraft_grow_workspace_size": _c_size,
              "treegraft_ngram_index_bytes": _c_size,
+             "treegraft_accept_sample_workspace_size": _c_size,
              "treegraft_tree_attn_workspace_size": _c_size,
              "treegraft_status_string": ctypes.c_char_p}
 
@@ -255,6 +260,47 @@ def accept(target_logits, token, parent, node_off, max_nodes, path_cap, ws, *, V
                                 int(path_cap), _ptr(path), _ptr(alen), _ptr(bonus), _ptr(ws),
                                 ws.numel(), _stream(stream))
     _check("treegraft_accept", st)
+    return path, alen, bonus
+
+
+def accept_sample_workspace(B: int, n_total: int, device) -> torch.Tensor:
+    """A zero-filled workspace for accept_sample (zeroed once; calls keep it
+    ready)."""
+    nbytes = int(lib().treegraft_accept_sample_workspace_size(int(B), int(n_total)))
+    if nbytes == 0:
+        raise ValueError("accept_sample workspace: invalid sizes")
+    return torch.zeros(nbytes, dtype=torch.uint8, device=device)
+
+
+def accept_sample(target_logits, token, parent, node_off, max_nodes, path_cap, u, temperature,
+                  ws, *, V=None, out=None, stream=None):
+    """Stochastic verification at temperature > 0 with the caller's uniforms
+    u fp32 [n_total, 2].  Returns (path [B, path_cap], accept_len [B],
+    bonus [B])."""
+    if target_logits.dim() != 2 or target_logits.stride(1) != 1 or not target_logits.is_cuda:
+        raise ValueError("target_logits must be a 2-D CUDA tensor with unit column stride")
+    dt = _logit_dtype(target_logits)
+    for t, nm in ((parent, "parent"), (token, "token"), (node_off, "node_off")):
+        _need(t, torch.int32, nm)
+    _need(u, torch.float32, "u")
+    _need(ws, torch.uint8, "ws")
+    n_total = parent.shape[0]
+    if tuple(u.shape) != (n_total, 2):
+        raise ValueError("u must be [n_total, 2]")
+    B = node_off.shape[0] - 1
+    V = target_logits.shape[1] if V is None else int(V)
+    dev = parent.device
+    if out is None:
+        out = (torch.empty(B, path_cap, dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev))
+    path, alen, bonus = out
+    st = lib().treegraft_accept_sample(_ptr(target_logits), dt, V, target_logits.stride(0),
+                                       float(temperature), _ptr(token), _ptr(parent),
+                                       _ptr(node_off), B, int(max_nodes), n_total, _ptr(u),
+                                       int(path_cap), _ptr(path), _ptr(alen), _ptr(bonus),
+                                       _ptr(ws), ws.numel(), _stream(stream))
+    _check("treegraft_accept_sample", st)
     return path, alen, bonus
 
 

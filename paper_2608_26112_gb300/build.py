@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libtreegraft.so")
 SOURCES = ["api.cu", "tree_attn.cu", "topk.cu", "accept.cu", "rescore.cu", "accept_noalloc.cu",
-           "prune.cu", "grow.cu", "ngram.cu"]
+           "prune.cu", "grow.cu", "ngram.cu", "sample.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
           "--expt-relaxed-constexpr", "-Xptxas", "-warn-spills"]

@@ -387,6 +387,55 @@ int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld, co
 }
 
 
+size_t treegraft_accept_sample_workspace_size(int B, int n_total) {
+  if (B < 1 || n_total < 1) return 0;
+  return sample_ws_bytes(B, n_total);
+}
+
+int treegraft_accept_sample(const void* target_logits, int dtype, int V, int64_t ld,
+                            float temperature, const int32_t* token, const int32_t* parent,
+                            const int32_t* node_off, int B, int max_nodes, int n_total,
+                            const float* u, int path_cap, int32_t* path, int32_t* accept_len,
+                            int32_t* bonus, void* ws, size_t ws_bytes, void* stream) {
+  if (!target_logits || !token || !parent || !node_off || !u || !path || !accept_len || !bonus ||
+      !ws)
+    return TG_ERR_INVALID_ARG;
+  if (dtype != TG_BF16 && dtype != TG_F32) return TG_ERR_INVALID_ARG;
+  if (!(temperature > 0.f) || !std::isfinite(temperature)) return TG_ERR_INVALID_ARG;
+  if (B < 1 || V < 1 || ld < V || n_total < 1 || path_cap < 1 || max_nodes < 1 ||
+      max_nodes > TG_MAX_TREE_NODES || (long long)n_total > (long long)B * max_nodes)
+    return TG_ERR_INVALID_ARG;
+  if (ws_bytes < sample_ws_bytes(B, n_total) || !aligned16(ws)) return TG_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(target_logits) & (dtype == TG_BF16 ? 1 : 3)) != 0)
+    return TG_ERR_INVALID_ARG;  // elements must sit at their natural alignment
+  if (V > (dtype == TG_BF16 ? 262144 : 131072) || B > 65535) return TG_ERR_UNSUPPORTED;
+  const float scale = 1.4426950408889634f / temperature;
+  if (!std::isfinite(scale)) return TG_ERR_UNSUPPORTED;  // T below what fp32 can scale
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  SampleArgs a = {};
+  a.logits = target_logits;
+  a.is_bf16 = dtype == TG_BF16;
+  a.V = V;
+  a.ld = ld;
+  a.scale_log2 = scale;
+  a.token = token;
+  a.parent = parent;
+  a.node_off = node_off;
+  a.B = B;
+  a.n_total = n_total;
+  a.path_cap = path_cap;
+  a.u = u;
+  a.path = path;
+  a.accept_len = accept_len;
+  a.bonus = bonus;
+  a.status = st;
+  sample_ws_carve(a, ws, B, n_total);
+  return launch_accept_sample(a, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? TG_OK
+             : TG_ERR_CUDA;
+}
+
 size_t treegraft_ngram_index_bytes(int B, int n_tokens, int max_n) {
   if (!ngram_shape_ok(B, n_tokens, max_n) || !ngram_shape_supported(n_tokens)) return 0;
   return ngram_layout(B, n_tokens, max_n).total;

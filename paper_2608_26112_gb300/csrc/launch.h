@@ -89,6 +89,31 @@ struct AcceptArgs {
 };
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s);
 
+struct SampleArgs {
+  const void* logits;
+  int is_bf16;
+  int V;
+  int64_t ld;
+  float scale_log2;  // log2(e) / T
+  const int32_t* token;
+  const int32_t* parent;
+  const int32_t* node_off;
+  int B, n_total, path_cap;
+  const float* u;  // [n_total, 2]
+  int32_t* path;
+  int32_t* accept_len;
+  int32_t* bonus;
+  // workspace (sample_ws_carve)
+  float2* stat;      // [n_total] row (max, sum of 2^((l - max) * scale_log2))
+  int32_t* flag;     // [n_total] child accepted by its parent's rule
+  int32_t* astar;    // [B]
+  int32_t* tickets;  // [B], zero between calls
+  int* status;
+};
+size_t sample_ws_bytes(int B, int n_total);
+void sample_ws_carve(SampleArgs& a, void* ws, int B, int n_total);
+cudaError_t launch_accept_sample(const SampleArgs& a, cudaStream_t s);
+
 struct PruneArgs {
   const float* score;
   const int32_t* parent;

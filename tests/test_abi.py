@@ -199,3 +199,22 @@ def test_ngram_rejects_bad_args_on_host(lib):
     assert grow(cap=20) == 1                 # 5 + 4 * 4 children do not fit
     assert grow(pool_lo=5) == 1
     assert grow(cap=2048, n=5) == 2          # beyond TG_MAX_GROW_NODES
+
+
+def test_accept_sample_rejects_bad_args_on_host(lib):
+    fake = ctypes.c_void_p(0x1000)
+    need = lib.treegraft_accept_sample_workspace_size(2, 100)
+    assert need == 1024 + 512 + 256 + 256
+    assert lib.treegraft_accept_sample_workspace_size(0, 100) == 0
+
+    def call(T=1.0, u=fake, nbytes=need, V=100, max_nodes=64, B=2):
+        return lib.treegraft_accept_sample(fake, 0, V, V, T, fake, fake, fake, B, max_nodes, 100,
+                                           u, 8, fake, fake, fake, fake, nbytes, NULL)
+    assert call(T=0.0) == 1
+    assert call(T=-1.0) == 1
+    assert call(T=float("inf")) == 1
+    assert call(T=1e-39) == 2                     # log2(e) / T overflows fp32
+    assert call(u=NULL) == 1
+    assert call(nbytes=need - 1) == 1
+    assert call(max_nodes=300) == 1
+    assert call(V=300000) == 2
