@@ -108,7 +108,8 @@ def build_sets(R, seed, dev):
                  prefix_len=t(wl["prefix_len"]), parent=t(wl["parent"]), token=t(wl["token"]),
                  node_off=t(wl["node_off"]), logits=bf(wl["logits"]),
                  target=bf(wl["target_logits"]), parent_score=t(wl["parent_score"]),
-                 weak_edge=t(wl["weak_edge"]), visited=t(wl["visited"]), strong=strong)
+                 weak_edge=t(wl["weak_edge"]), visited=t(wl["visited"]), strong=strong,
+                 u=t(rng.random((len(wl["parent"]), 2)).astype(np.float32)))
         sets.append(d)
         wl.pop("strong_lp", None)
         host.append(wl)
@@ -133,6 +134,7 @@ def alloc_outputs(d, sh, dev):
         alen=torch.empty(1, dtype=torch.int32, device=dev),
         bonus=torch.empty(1, dtype=torch.int32, device=dev),
         ws=tg.accept_workspace(1, n, dev),
+        sws=tg.accept_sample_workspace(1, n, dev),
         attn_ws=torch.zeros(max(16, tg.tree_attn_workspace_size(
             1, n, d["q"].shape[1], d["k"].shape[1], d["q"].shape[2])), dtype=torch.uint8,
             device=dev))
@@ -153,9 +155,15 @@ def call(name, d, o, sh):
     elif name == "accept":
         tg.accept(d["target"], d["token"], d["parent"], d["node_off"], n, n, o["ws"],
                   out=(o["path"], o["alen"], o["bonus"]))
+    elif name == "accept_sample":
+        tg.accept_sample(d["target"], d["token"], d["parent"], d["node_off"], n, n, d["u"],
+                         SAMPLE_T, o["sws"], out=(o["path"], o["alen"], o["bonus"]))
 
 
 KERNELS = ["tree_attn", "expand_topk", "rescore_select", "accept"]
+# timed beside the step: verification at temperature SAMPLE_T instead of 0
+BESIDE = ["accept_sample"]
+SAMPLE_T = 1.0
 
 
 def step(d, o, sh):
@@ -733,7 +741,7 @@ def ours_arm(args):
     singles = [capture(lambda r=r: step(sets[r], outs[r], sh), stream) for r in range(R)]
     per_kernel_graphs = {name: capture(lambda name=name: [call(name, sets[r], outs[r], sh)
                                                          for r in range(R)], stream)
-                         for name in KERNELS}
+                         for name in KERNELS + BESIDE}
     for _ in range(3):
         cycle.replay()
     torch.cuda.synchronize()
@@ -781,6 +789,12 @@ def ours_arm(args):
                          "hbm_frac": b / kt[name] / 1e9 / hbm}
         if f:
             kernels[name]["TFLOPs"] = f / kt[name] / 1e12
+    b = costs["accept"][0] + host[0]["shape"]["V"] * 2
+    kernels["accept_sample"] = {"us": kt["accept_sample"] * 1e6, "bytes": b,
+                                "GBps": b / kt["accept_sample"] / 1e9,
+                                "hbm_frac": b / kt["accept_sample"] / 1e9 / hbm,
+                                "temperature": SAMPLE_T, "launches": 2, "in_step": False,
+                                "note": "verification at T > 0: every node row, then row a*"}
     kernels["global_prune"] = prune
     kernels["grow_loop"] = grow
     kernels["ngram_drafter"] = ngram
