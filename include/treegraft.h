@@ -357,10 +357,12 @@ int treegraft_grow_step(int mode, const void* logits, int dtype, int V, int64_t 
  * draw at v).  temperature > 0 (fp32 must be able to hold log2(e) / T).
  * ws: treegraft_accept_sample_workspace_size(B, n_total) bytes, 16-byte
  * aligned, ZEROED before its first use (per-tree tickets, reset by every
- * call).  Two launches: per node row the (max, sum) and every child's
- * decision, and the walk in the CTA that finishes a tree's rows; then row
- * a* per tree for the bonus draw.  The comparisons are taken in fp32, so a
- * draw within a few ulps of a threshold may fall either way.
+ * call).  One launch: per node row, the masses 2^((l - max) log2(e) / T)
+ * in 44-bit fixed point (exact, order-free sums), every child's decision
+ * and the bonus draw the row would give if the walk ended there; the CTA
+ * that finishes a tree's rows walks it.  The masses carry the rounding of
+ * the exponential and of the fixed point, so a draw within about 1e-7 of
+ * a threshold may fall either way.
  * Errors: TG_ERR_INVALID_ARG, TG_ERR_UNSUPPORTED (V too large, B > 65535,
  * T too small), TG_ERR_CUDA; a malformed tree sets TG_ERR_DEVICE_TREE and a
  * token outside [0, V) or a path longer than path_cap TG_ERR_DEVICE_INDEX

@@ -104,9 +104,8 @@ struct SampleArgs {
   int32_t* accept_len;
   int32_t* bonus;
   // workspace (sample_ws_carve)
-  float2* stat;      // [n_total] row (max, sum of 2^((l - max) * scale_log2))
   int32_t* flag;     // [n_total] child accepted by its parent's rule
-  int32_t* astar;    // [B]
+  int32_t* bcand;    // [n_total] bonus token if the walk ends at that node
   int32_t* tickets;  // [B], zero between calls
   int* status;
 };

@@ -204,7 +204,7 @@ def test_ngram_rejects_bad_args_on_host(lib):
 def test_accept_sample_rejects_bad_args_on_host(lib):
     fake = ctypes.c_void_p(0x1000)
     need = lib.treegraft_accept_sample_workspace_size(2, 100)
-    assert need == 1024 + 512 + 256 + 256
+    assert need == 512 + 512 + 256          # flags, bonus candidates, tickets
     assert lib.treegraft_accept_sample_workspace_size(0, 100) == 0
 
     def call(T=1.0, u=fake, nbytes=need, V=100, max_nodes=64, B=2):
