@@ -94,26 +94,29 @@ __device__ __forceinline__ bool same_gram(const int32_t* tok, int p, int j, int 
   return true;
 }
 
+// One thread per (position j, order n): the n-gram ending at j hashed from
+// its n tokens (independent loads), then inserted into table n.
 __global__ void __launch_bounds__(256) ngram_insert_kernel(NgramArgs a) {
   const uint32_t mask = (uint32_t)a.T - 1u;
-  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < a.n_tokens; j += gridDim.x * blockDim.x) {
+  const long long items = (long long)a.n_tokens * a.max_n;
+  for (long long it = blockIdx.x * (long long)blockDim.x + threadIdx.x; it < items;
+       it += (long long)gridDim.x * blockDim.x) {
+    const int j = (int)(it / a.max_n), i = (int)(it - (long long)j * a.max_n);  // order i + 1
     const int b = seq_of(a.seq, a.B, j);
     const int lo = max(a.seq[b], 0), hi = min(a.seq[b + 1], a.n_tokens);
-    if (j < lo || j >= hi) continue;  // only with a malformed seq (status raised)
+    if (j < lo || j >= hi || j - i < lo) continue;  // outside the prompt (or a malformed seq)
     uint32_t h = hash_seed(b);
-    for (int i = 0; i < a.max_n && j - i >= lo; ++i) {
-      h = hash_step(h, a.tok[j - i]);
-      int32_t* tab = a.tab + (size_t)i * a.T;
-      uint32_t slot = h & mask;
-      for (int it = 0; it < a.T; ++it) {  // an empty slot always exists (load <= 1/2)
-        const int old = atomicCAS(tab + slot, -1, j);
-        if (old == -1 || same_gram(a.tok, old, j, i + 1, lo, hi)) {
-          if (old != -1) atomicMax(tab + slot, j);
-          if (i == 0) atomicAdd(a.cnt + slot, 1);
-          break;
-        }
-        slot = (slot + 1u) & mask;
+    for (int k = 0; k <= i; ++k) h = hash_step(h, a.tok[j - k]);
+    int32_t* tab = a.tab + (size_t)i * a.T;
+    uint32_t slot = h & mask;
+    for (int probe = 0; probe < a.T; ++probe) {  // an empty slot always exists (load <= 1/2)
+      const int old = atomicCAS(tab + slot, -1, j);
+      if (old == -1 || same_gram(a.tok, old, j, i + 1, lo, hi)) {
+        if (old != -1) atomicMax(tab + slot, j);
+        if (i == 0) atomicAdd(a.cnt + slot, 1);
+        break;
       }
+      slot = (slot + 1u) & mask;
     }
   }
 }
@@ -160,7 +163,8 @@ __device__ __forceinline__ int ngram_probe(const NgramArgs& a, int lo, int hi,
 // precede its child is the caller's to catch).  Returns the hit word
 // (n << 27 | position) or -1 (query shorter than n, or no occurrence).
 template <typename TreeRead>
-__device__ __forceinline__ int ngram_order_hit(const NgramArgs& a, int b, int v, int n, int clen,
+__device__ __forceinline__ int ngram_order_hit(const NgramArgs& a, int b, int v, int n,
+                                               const int32_t* ctxp, int clen,
                                                TreeRead&& tree) {
   int32_t q[kNgramMaxN];
   int w = v, ci = clen - 1;
@@ -175,7 +179,7 @@ __device__ __forceinline__ int ngram_order_hit(const NgramArgs& a, int b, int v,
         tree(w, x, pa);
         w = pa;
       } else if (ci >= 0) {
-        x = __ldg(a.ctx + (size_t)b * a.max_n + ci);
+        x = ctxp[ci];
         --ci;
       } else {
         full = false;
@@ -217,7 +221,8 @@ __global__ void __launch_bounds__(256) ngram_draft_kernel(NgramArgs a) {
   bool bad = false;
   int hit = -1;
   if (lane < a.max_n) {
-    hit = ngram_order_hit(a, b, v, lane + 1, clen, [&](int w, int32_t& x, int& pa) {
+    hit = ngram_order_hit(a, b, v, lane + 1, a.ctx + (size_t)b * a.max_n, clen,
+                          [&](int w, int32_t& x, int& pa) {
       x = __ldg(a.token + base + w);
       pa = __ldg(a.parent + base + w);
       if (pa < 0 || pa >= w) {  // parents come before children
@@ -271,12 +276,16 @@ __global__ void __launch_bounds__(kGrowThreads) ngram_grow_kernel(NgramArgs a) {
   __shared__ uint64_t key_s[kGrowThreads];
   __shared__ int front_s[kGrowThreads];
   __shared__ int best_s[kGrowThreads];
+  __shared__ int32_t ctx_s[kNgramMaxN];
   const int b = blockIdx.x;
   const int tid = threadIdx.x, nth = blockDim.x;
   const int n = a.n, lo = a.pool_lo, nf = min(a.W, n - lo);
   const size_t base = (size_t)b * a.cap;
   pdl_launch_dependents();
   pdl_wait();
+  // the committed context and the fallback position load with the tree
+  if (tid < a.max_n) ctx_s[tid] = __ldg(a.ctx + (size_t)b * a.max_n + tid);
+  const int fb = __ldg(a.fbp + b);
   int bad = 0;
   for (int v = tid; v < n; v += nth) {
     const int p = a.parent[base + v];
@@ -306,14 +315,13 @@ __global__ void __launch_bounds__(kGrowThreads) ngram_grow_kernel(NgramArgs a) {
   __syncthreads();
   for (int item = tid; item < nf * a.max_n; item += nth) {
     const int i = item / a.max_n, ord = item - i * a.max_n + 1;
-    const int hit = ngram_order_hit(a, b, front_s[i], ord, clen, [&](int w, int32_t& x, int& pa) {
+    const int hit = ngram_order_hit(a, b, front_s[i], ord, ctx_s, clen, [&](int w, int32_t& x, int& pa) {
       x = tok_s[w];
       pa = par_s[w];
     });
     if (hit >= 0) atomicMax(&best_s[i], hit);
   }
   __syncthreads();
-  const int fb = __ldg(a.fbp + b);
   const int m = a.m;
   for (int item = tid; item < nf * m; item += nth) {
     const int i = item / m, c = item - i * m;
@@ -394,7 +402,7 @@ void ngram_carve(NgramArgs& a, void* index, int B, int n_tokens, int max_n) {
 cudaError_t launch_ngram_build(const NgramArgs& a, cudaStream_t s) {
   const size_t span = std::max((size_t)a.max_n * a.T, (size_t)std::max(a.n_tokens, a.B + 1));
   ngram_init_kernel<<<grid_for(span), 256, 0, s>>>(a);
-  ngram_insert_kernel<<<grid_for(a.n_tokens), 256, 0, s>>>(a);
+  ngram_insert_kernel<<<grid_for((size_t)a.n_tokens * a.max_n), 256, 0, s>>>(a);
   ngram_fallback_kernel<<<grid_for(a.T), 256, 0, s>>>(a, 0);
   ngram_fallback_kernel<<<grid_for(a.T), 256, 0, s>>>(a, 1);
   return cudaGetLastError();
