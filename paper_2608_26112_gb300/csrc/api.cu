@@ -206,7 +206,7 @@ int treegraft_expand_topk(const void* logits, int dtype, int logit_rows, int V, 
   if (k > TG_MAX_TOPK || V > (dtype == TG_BF16 ? 262144 : 131072)) return TG_ERR_UNSUPPORTED;
   int* st = status_ptr();
   if (!st) return TG_ERR_CUDA;
-  TopkArgs a;
+  TopkArgs a = {};
   a.logits = logits;
   a.is_bf16 = dtype == TG_BF16;
   a.logit_rows = logit_rows;

@@ -9,17 +9,17 @@
 // P is always a prefix [0, |P|) of the node ids - P only grows at middle
 // steps, where it becomes P u (V \ P) = V, and nodes are only ever appended.
 //
-// Small step (a = 0), three launches:
+// Small step (a = 0), two launches:
 //   grow_select   Top_W of the pool by (s desc, id asc) -> frontier F, and the
 //                 expansion rows with their path scores;
 //   expand_topk   Top_m of each frontier row of the small drafter's table
-//                 (log-softmax, token ids, fp32(s(v) + p(u)));
-//   grow_append   children appended at n, n + 1, ... in frontier order, then
-//                 child rank.
-// Middle step (a = 1), three launches:
-//   grow_prep     the pool's rows of the middle drafter's table;
+//                 (log-softmax, token ids, fp32(s(v) + p(u))), the children
+//                 appended straight into the tree at n, n + 1, ... in
+//                 frontier order, then child rank.
+// Middle step (a = 1), two launches:
 //   expand_topk   log-sum-exp and Top_m of every pool row (the drafter's
-//                 forward over C, whose logits are then reused for F);
+//                 forward over C, whose logits are then reused for F), the
+//                 rows of each tree's pool [pool_lo, n) mapped in the kernel;
 //   grow_select   caches each pool row's lse, rescores every non-root pool
 //                 node p(v) = l_m[pa(v), token(v)] - lse_m[pa(v)], recomputes
 //                 s root-first, takes Top_W of the pool and appends the
@@ -41,20 +41,6 @@ __device__ __forceinline__ float logit_at(const void* logits, int is_bf16, int64
     return __uint_as_float((uint32_t)h << 16);
   }
   return reinterpret_cast<const float*>(logits)[row * (size_t)ld + col];
-}
-
-// Middle step: the pool's rows of the drafter table for expand_topk (row
-// b * |C| + j is node pool_lo + j of tree b) with zero parent scores (the
-// children's scores are made from the rescored s in grow_select).
-__global__ void __launch_bounds__(256) grow_prep_kernel(GrowArgs a) {
-  pdl_launch_dependents();
-  pdl_wait();
-  const int nc = a.n - a.pool_lo;
-  const int b = blockIdx.y;
-  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < nc; j += gridDim.x * blockDim.x) {
-    a.ws_row[(size_t)b * nc + j] = b * a.cap + a.pool_lo + j;
-    a.ws_ps[(size_t)b * nc + j] = 0.f;
-  }
 }
 
 __global__ void __launch_bounds__(kGrowThreads) grow_select_kernel(GrowArgs a) {
@@ -164,26 +150,6 @@ __global__ void __launch_bounds__(kGrowThreads) grow_select_kernel(GrowArgs a) {
   }
 }
 
-// Small step: children of the frontier from expand_topk's outputs (row
-// b * |F| + i is frontier node i of tree b; its scores are fp32(s(v) + p(u))).
-__global__ void __launch_bounds__(256) grow_append_kernel(GrowArgs a) {
-  pdl_launch_dependents();
-  pdl_wait();
-  const int nf = min(a.W, a.n - a.pool_lo), m = a.m;
-  const int b = blockIdx.y;
-  const size_t base = (size_t)b * a.cap;
-  for (int item = blockIdx.x * blockDim.x + threadIdx.x; item < nf * m;
-       item += gridDim.x * blockDim.x) {
-    const int i = item / m;
-    const size_t src = (size_t)b * nf * m + item;
-    const size_t u = base + a.n + item;
-    a.parent[u] = a.frontier[(size_t)b * a.W + i];
-    a.token[u] = a.ws_tok[src];
-    a.edge[u] = a.ws_lp[src];
-    a.score[u] = a.ws_sc[src];
-  }
-}
-
 cudaError_t launch_pdl(const void* fn, dim3 grid, dim3 block, const GrowArgs& a, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
@@ -228,29 +194,34 @@ cudaError_t launch_grow_step(const GrowArgs& a, cudaStream_t s) {
   t.logit_rows = a.B * a.cap;
   t.V = a.V;
   t.ld = a.ld;
-  t.row_idx = a.ws_row;
-  t.parent_score = a.ws_ps;
   t.k = a.m;
-  t.tok = a.ws_tok;
-  t.logprob = a.ws_lp;
-  t.score = a.ws_sc;
   t.status = a.status;
+  t.gcap = a.cap;
   const dim3 sel_grid(a.B), sel_block((unsigned)((a.n + 31) / 32 * 32));
   cudaError_t e;
   if (a.mode == 0) {
     e = launch_pdl(reinterpret_cast<const void*>(grow_select_kernel), sel_grid, sel_block, a, s);
     if (e != cudaSuccess) return e;
+    // row b * nf + i = frontier node i of tree b (ws_row), its children
+    // appended to the tree
     t.rows = a.B * nf;
-    t.lse_out = nullptr;
-    e = launch_expand_topk(t, s);
-    if (e != cudaSuccess) return e;
-    const dim3 grid((unsigned)((nf * a.m + 255) / 256), a.B);
-    return launch_pdl(reinterpret_cast<const void*>(grow_append_kernel), grid, dim3(256), a, s);
+    t.row_idx = a.ws_row;
+    t.parent_score = a.ws_ps;
+    t.gdiv = nf;
+    t.app_n = a.n;
+    t.app_parent = a.parent;
+    t.app_token = a.token;
+    t.app_edge = a.edge;
+    t.app_score = a.score;
+    return launch_expand_topk(t, s);
   }
-  const dim3 grid((unsigned)((nc + 255) / 256), a.B);
-  e = launch_pdl(reinterpret_cast<const void*>(grow_prep_kernel), grid, dim3(256), a, s);
-  if (e != cudaSuccess) return e;
+  // row b * nc + j = pool node pool_lo + j of tree b; zero parent scores (the
+  // children's scores come from the rescored s in grow_select)
   t.rows = a.B * nc;
+  t.gdiv = nc;
+  t.goff = a.pool_lo;
+  t.tok = a.ws_tok;
+  t.logprob = a.ws_lp;
   t.lse_out = a.ws_lse;
   e = launch_expand_topk(t, s);
   if (e != cudaSuccess) return e;

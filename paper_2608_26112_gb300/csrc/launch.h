@@ -49,6 +49,18 @@ struct TopkArgs {
   float* score;
   float* lse_out;
   int* status;
+  // Tree batches (the grow step).  Without row_idx and with gdiv > 0,
+  // logical row i reads physical row (i / gdiv) * gcap + goff + i % gdiv
+  // (the pool rows of each tree).  With app_token set, row i = tree i / gdiv,
+  // frontier slot i % gdiv, and its children are appended to the tree
+  // arrays at (i / gdiv) * gcap + app_n + (i % gdiv) * k + rank, with
+  // parent = the physical row - (i / gdiv) * gcap.
+  int gdiv, gcap, goff, app_n;
+  int32_t* app_parent;
+  int32_t* app_token;
+  float* app_edge;
+  float* app_score;
+  int row0;  // first logical row of this launch (grids of at most 65535 rows)
 };
 cudaError_t launch_expand_topk(const TopkArgs& a, cudaStream_t s);
 int scan_cluster_size(int V, int is_bf16, int rows, int num_sms);

@@ -209,13 +209,15 @@ __device__ __noinline__ void exact_topk_fallback(const T* __restrict__ rowp, int
   __syncthreads();
 }
 
-template <typename T, bool kAligned>
+// kTree: the tree-batch row mapping and the append of children (grow step),
+// compiled out of the plain kernel.
+template <typename T, bool kAligned, bool kTree>
 __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a) {
   __shared__ TopkSmem sm;
   cg::cluster_group cluster = cg::this_cluster();
   const int C = (int)cluster.num_blocks();
   const int crank = (int)cluster.block_rank();
-  const int row = blockIdx.y;
+  const int row = a.row0 + (int)blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int k = a.k;
   const int V = a.V;
@@ -226,7 +228,12 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   pdl_wait();
   // physical row (uniform over the cluster: every CTA reads the same index)
   int r = row;
-  if (a.row_idx) r = a.row_idx[row];
+  if (a.row_idx) {
+    r = a.row_idx[row];
+  } else if (kTree && a.gdiv) {
+    const int bt = row / a.gdiv;
+    r = bt * a.gcap + a.goff + (row - bt * a.gdiv);
+  }
   if (r < 0 || r >= a.logit_rows) {
     if (crank == 0 && tid == 0) raise_status(a.status, kStIndex);
     return;
@@ -293,10 +300,19 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
     if (rank < k) {
       const float v = key_value(key);
       const float lp = (lse == NEG_INF) ? lse : (v - lse);
-      const size_t o = (size_t)row * k + rank;
-      a.tok[o] = (int32_t)key_index(key);
-      a.logprob[o] = lp;
-      if (a.score) a.score[o] = __fadd_rn(parent_score, lp);
+      if (kTree && a.app_token) {  // children appended to the tree (grow step)
+        const int bt = row / a.gdiv;
+        const size_t u = (size_t)bt * a.gcap + a.app_n + (size_t)(row - bt * a.gdiv) * k + rank;
+        a.app_parent[u] = r - bt * a.gcap;
+        a.app_token[u] = (int32_t)key_index(key);
+        a.app_edge[u] = lp;
+        a.app_score[u] = __fadd_rn(parent_score, lp);
+      } else {
+        const size_t o = (size_t)row * k + rank;
+        a.tok[o] = (int32_t)key_index(key);
+        a.logprob[o] = lp;
+        if (a.score) a.score[o] = __fadd_rn(parent_score, lp);
+      }
       if (rank == 0 && a.lse_out) a.lse_out[row] = lse;
     }
   }
@@ -304,7 +320,8 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
 
 template <typename T, bool kAligned>
 cudaError_t launch_topk_t(const TopkArgs& a, int C, cudaStream_t s) {
-  auto kern = expand_topk_kernel<T, kAligned>;
+  auto kern = (a.gdiv || a.app_token) ? expand_topk_kernel<T, kAligned, true>
+                                      : expand_topk_kernel<T, kAligned, false>;
   if (C > 8) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
@@ -313,17 +330,7 @@ cudaError_t launch_topk_t(const TopkArgs& a, int C, cudaStream_t s) {
     TopkArgs b = a;
     const int nr = min(65535, a.rows - r0);
     b.rows = nr;
-    if (b.row_idx) {
-      b.row_idx += r0;
-    } else {
-      b.logits = static_cast<const char*>(a.logits) + (size_t)r0 * (size_t)a.ld * (a.is_bf16 ? 2 : 4);
-      b.logit_rows = a.logit_rows - r0;
-    }
-    if (b.parent_score) b.parent_score += r0;
-    b.tok += (size_t)r0 * a.k;
-    b.logprob += (size_t)r0 * a.k;
-    if (b.score) b.score += (size_t)r0 * a.k;
-    if (b.lse_out) b.lse_out += r0;
+    b.row0 = r0;  // the kernel indexes rows, parent scores and outputs by r0 + blockIdx.y
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(C, nr, 1);
     cfg.blockDim = dim3(kScanThreads, 1, 1);
