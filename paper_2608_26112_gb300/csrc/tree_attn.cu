@@ -382,6 +382,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kBN, false);
       constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, true);
       const uint32_t tmem_O = tmem + 256u;
+      // Operand descriptors as base + offset / 16: the start-address field
+      // (bits 0-13, 16-byte units) of a base descriptor plus the byte offset
+      // of the operand, exact while the address stays below 256 KB.  One
+      // thread issues every product, so the few integer ops per MMA instead
+      // of a full descriptor build keep the tensor pipe fed.
+      const uint64_t dq0 = smem_desc_sw128(q_base, 16, 1024);
+      const uint64_t dk0 = smem_desc_sw128(k_base, 16, 1024);
+      const uint64_t dv0 = smem_desc_sw128(v_base, kRegion, 1024);
       bool ok = mbar_wait(bar(BAR_Q_FULL), 0);
       for (int it = 0; ok && it <= nt; ++it) {
         if (it < nt) {
@@ -392,12 +400,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (ok && it >= 2) ok = mbar_wait(bar(BAR_O_DONE + st), ((it - 2) >> 1) & 1);
           if (!ok) break;
           tc_fence_after();
+          const uint64_t dk = dk0 + (uint64_t)((st * L::kKVBytes) >> 4);
+          const uint32_t ts = tmem + (uint32_t)(st * 128);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t qa = q_base + (kk >> 2) * kRegion + (kk & 3) * 32;
-            const uint32_t ka = k_base + st * L::kKVBytes + (kk >> 2) * kRegion + (kk & 3) * 32;
-            tc_mma_f16(tmem + (uint32_t)(st * 128), smem_desc_sw128(qa, 16, 1024),
-                       smem_desc_sw128(ka, 16, 1024), kIdS, kk > 0 ? 1u : 0u);
+            const uint32_t o = (uint32_t)((kk >> 2) * kRegion + (kk & 3) * 32) >> 4;
+            tc_mma_f16(ts, dq0 + o, dk + o, kIdS, kk > 0 ? 1u : 0u);
           }
           tc_commit(bar(BAR_S_FULL + st));
           tc_commit(bar(BAR_K_EMPTY + st));
@@ -407,13 +415,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = mbar_wait(bar(BAR_P_FULL), jt & 1) && mbar_wait(bar(BAR_V_FULL + sp), (jt >> 1) & 1);
           if (!ok) break;
           tc_fence_after();
+          const uint64_t dv = dv0 + (uint64_t)((sp * L::kKVBytes) >> 4);
+          const uint32_t pa = tmem + (uint32_t)(sp * 128);
+          const uint32_t acc0 = jt > 0 ? 1u : 0u;
 #pragma unroll
           for (int kk = 0; kk < kBN / 16; ++kk) {
             // P(jt) in S buffer jt&1: 16 keys per MMA = 8 TMEM columns
-            const uint32_t pa = tmem + (uint32_t)(sp * 128 + kk * 8);
-            const uint32_t va = v_base + sp * L::kKVBytes + kk * 16 * 128;
-            tc_mma_f16_ts(tmem_O, pa, smem_desc_sw128(va, kRegion, 1024), kIdO,
-                          (jt > 0 || kk > 0) ? 1u : 0u);
+            tc_mma_f16_ts(tmem_O, pa + (uint32_t)(kk * 8), dv + (uint64_t)((kk * 16 * 128) >> 4),
+                          kIdO, kk > 0 ? 1u : acc0);
           }
           tc_commit(bar(BAR_O_DONE + sp));
           tc_commit(bar(BAR_V_EMPTY + sp));
