@@ -116,6 +116,46 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
                : "memory");
 }
 
+// Paired fp32 arithmetic of sm_100-class SMs: one instruction for two
+// independent round-to-nearest operations (the same results as two scalar
+// ones), and the three-input max.
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;"
+      : "=l"(d)
+      : "l"(*reinterpret_cast<const uint64_t*>(&a)), "l"(*reinterpret_cast<const uint64_t*>(&b)),
+        "l"(*reinterpret_cast<const uint64_t*>(&c)));
+  return *reinterpret_cast<float2*>(&d);
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;"
+      : "=l"(d)
+      : "l"(*reinterpret_cast<const uint64_t*>(&a)), "l"(*reinterpret_cast<const uint64_t*>(&b)));
+  return *reinterpret_cast<float2*>(&d);
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+// max of 64 values as four independent chains of three-input maxima
+__device__ __forceinline__ float max64(const float (&s)[64]) {
+  float ma = s[0], mb = s[2], mc = s[4], md = s[6];
+  ma = fmaxf(ma, s[1]);
+  mb = fmaxf(mb, s[3]);
+  mc = fmaxf(mc, s[5]);
+  md = fmaxf(md, s[7]);
+#pragma unroll
+  for (int c = 8; c < 64; c += 8) {
+    ma = max3(ma, s[c], s[c + 1]);
+    mb = max3(mb, s[c + 2], s[c + 3]);
+    mc = max3(mc, s[c + 4], s[c + 5]);
+    md = max3(md, s[c + 6], s[c + 7]);
+  }
+  return max3(ma, mb, fmaxf(mc, md));
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
@@ -497,19 +537,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld32f(ts, *reinterpret_cast<float(*)[32]>(&s[0]));
         tmem_ld32f(ts + 32, *reinterpret_cast<float(*)[32]>(&s[32]));
         tc_wait_ld();
-        if (key0 + 64 <= P) {
-#pragma unroll
-          for (int c = 0; c < 64; ++c) mx = fmaxf(mx, s[c]);
-        } else {
+        if (key0 + 64 > P) {
           const uint32_t mw0 = mask_word(anc, key0 - P);
           const uint32_t mw1 = mask_word(anc, key0 + 32 - P);
 #pragma unroll
           for (int c = 0; c < 64; ++c) {
             const bool vis = (((c < 32) ? mw0 : mw1) >> (c & 31)) & 1u;
             s[c] = vis ? s[c] : NEG_INF;
-            mx = fmaxf(mx, s[c]);
           }
         }
+        mx = max64(s);
       }
       // row max over both halves (double-buffered by tile parity)
       float* rm = red_max + st * 2 * kBM;
@@ -525,15 +562,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float m_use = (m_new == NEG_INF) ? 0.f : m_new;
       const float nb = -m_use * sl2;
       const float corr = ex2(fmaf(m_run, sl2, nb));
-      float rs0 = 0.f, rs1 = 0.f;
+      const float2 sl2v = make_float2(sl2, sl2), nbv = make_float2(nb, nb);
+      // row sum in eight independent chains (four paired accumulators)
+      float2 racc[4];
 #pragma unroll
       for (int c = 0; c < 64; c += 2) {
-        s[c] = ex2(fmaf(s[c], sl2, nb));
-        s[c + 1] = ex2(fmaf(s[c + 1], sl2, nb));
-        rs0 += s[c];
-        rs1 += s[c + 1];
+        const float2 x = fma2(make_float2(s[c], s[c + 1]), sl2v, nbv);
+        s[c] = ex2(x.x);
+        s[c + 1] = ex2(x.y);
+        const float2 e = make_float2(s[c], s[c + 1]);
+        racc[(c >> 1) & 3] = c < 8 ? e : add2(racc[(c >> 1) & 3], e);
       }
-      l_run = l_run * corr + (rs0 + rs1);
+      const float2 rsum = add2(add2(racc[0], racc[1]), add2(racc[2], racc[3]));
+      l_run = l_run * corr + (rsum.x + rsum.y);
       if (it > 0 && __any_sync(0xffffffffu, m_new > m_run)) {
         // PV(it-1) must finish before O is rescaled
         ok = __all_sync(0xffffffffu, observe(it));
