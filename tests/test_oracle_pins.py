@@ -653,6 +653,24 @@ def test_grow_tree_all_small_is_single_drafter_construction():
         assert abs(score[v] - path) < 1e-5
 
 
+def test_grow_tree_frontier_ties_go_to_the_lower_node_id():
+    """Top_W ranks by (score desc, node id asc).  The root's children come
+    from a row whose four best logits are equal, so they carry equal scores;
+    the next small step's frontier of W = 2 is the two with the lowest ids,
+    and a middle step over the same tree keeps that order among equals."""
+    small = np.zeros((32, 8), np.float32)
+    small[0, [2, 4, 5, 7]] = 3.0
+    middle = np.zeros((32, 8), np.float32)
+    par, tok, edge, score, vis, fr = O.grow_tree([0, 0], 2, 4, small, middle)
+    assert tok[1:5].tolist() == [2, 4, 5, 7]
+    assert len(set(score[1:5].tolist())) == 1
+    assert fr == [[0], [1, 2]]
+    # middle step: every row uniform, so all non-root scores tie; the root
+    # (score 0, the largest) comes first, then the lowest ids
+    par, tok, edge, score, vis, fr = O.grow_tree([0, 1], 3, 4, small, middle)
+    assert fr[1] == [0, 1, 2]
+
+
 def test_grow_tree_middle_first_step_expands_the_root():
     rng = synth.make_rng(72)
     small = synth.normal_f32(rng, (32, 16), 2.0)
