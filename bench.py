@@ -694,11 +694,13 @@ def reference_arm(args):
     if rank != 0:
         return
     per_step_min = 0.0
-    steps, sec = run_cpu_oracle(max(1, args.steps if args.steps < 50 else 5),
-                                min(args.warmup, 1), per_step_min, 120.0)
+    # bounded: at most 5 timed steps and 3 warm-up steps of the oracle
+    warm = min(args.warmup, 3)
+    steps, sec = run_cpu_oracle(max(1, args.steps if args.steps < 50 else 5), warm,
+                                per_step_min, 120.0)
     v = steps / sec
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "steps/s",
-            "n_gpus": args.gpus, "steps": steps, "warmup": min(args.warmup, 1),
+            "n_gpus": args.gpus, "steps": steps, "warmup": warm,
             "ms_per_step": 1e3 * sec / steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": WORKLOAD, "note": "oracle (plain fp64 numpy) on host cores"},
