@@ -4,7 +4,8 @@ Each case plants one mistake in an in-memory copy of an oracle module: a
 dropped term, a wrong index, sign or tie rule, a transposed operand, an
 off-by-one.  The case points the pin tests (tests/test_oracle_pins.py,
 test_oracle_sample.py, test_oracle_ngram.py) at that copy and runs them with
-every parametrisation.  At least one pin must fail.  The oracle files are
+every parametrisation; the oracle modules built on the mutated one see the
+copy too.  At least one pin must fail.  The oracle files are
 only read, never modified.  CPU only."""
 import inspect
 import os
@@ -12,15 +13,20 @@ import types
 
 import pytest
 
+from oracle import ngram_oracle, sample_oracle
 from tests import test_oracle_ngram, test_oracle_pins, test_oracle_sample
 
 ORACLE_DIR = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "oracle")
 
-# (oracle module, pin module, the pin module's name for the oracle module)
-TARGETS = {
-    "treegraft_oracle": (test_oracle_pins, "O"),
-    "sample_oracle": (test_oracle_sample, "S"),
-    "ngram_oracle": (test_oracle_ngram, "NG"),
+PIN_MODULES = (test_oracle_pins, test_oracle_sample, test_oracle_ngram)
+
+# oracle module -> every (module, global name) through which it is used: the
+# pin modules and the oracle modules built on it
+USES = {
+    "treegraft_oracle": ((test_oracle_pins, "O"), (test_oracle_sample, "O"),
+                         (test_oracle_ngram, "O"), (sample_oracle, "O"), (ngram_oracle, "T")),
+    "sample_oracle": ((test_oracle_sample, "S"),),
+    "ngram_oracle": ((test_oracle_ngram, "NG"),),
 }
 
 # id: (oracle module, exact text, replacement)
@@ -110,7 +116,13 @@ MUTATIONS = {
                                         "F = sorted(C, key=lambda v: (-float(score[v]), -v))[:W]"),
     "grow-score-subtracts": ("treegraft_oracle", "score.append(np.float32(score[v] + lp))",
                              "score.append(np.float32(score[v] - lp))"),
+    "grow-ngram-score-subtracts": ("treegraft_oracle",
+                                   "score.append(np.float32(score[v] + np.float32(lp)))",
+                                   "score.append(np.float32(score[v] - np.float32(lp)))"),
     # stochastic verification
+    "sample-children-descending": ("sample_oracle",
+                                   "            for c in children[v]:\n                x = int(token[a + c])",
+                                   "            for c in children[v][::-1]:\n                x = int(token[a + c])"),
     "sample-residual-kept": ("sample_oracle", "                R -= p[x]\n",
                              "                pass\n"),
     "sample-accept-inverted": ("sample_oracle", "if lhs < p[x]:", "if lhs > p[x]:"),
@@ -130,6 +142,7 @@ MUTATIONS = {
                                          "return min(j for j, t in enumerate(prompt) if int(t) == best)"),
     "ngram-shortest-order-first": ("ngram_oracle", "for n in range(min(max_n, len(query)), 0, -1):",
                                    "for n in range(1, min(max_n, len(query)) + 1):"),
+    "ngram-query-repeats-root-token": ("ngram_oracle", "    while w != 0:\n", "    while w != -1:\n"),
     "ngram-path-reversed": ("ngram_oracle", "seq = [int(t) for t in ctx] + path[::-1]",
                             "seq = [int(t) for t in ctx] + path"),
     "ngram-window-from-the-start": ("ngram_oracle", "return seq[-max_n:]", "return seq[:max_n]"),
@@ -182,25 +195,30 @@ def _pin_calls(pins):
             yield name, fn, kw
 
 
+def _all_pin_calls():
+    for pins in PIN_MODULES:
+        yield from _pin_calls(pins)
+
+
 def test_every_pin_module_has_runnable_pins():
-    for module, (pins, _) in TARGETS.items():
-        assert sum(1 for _ in _pin_calls(pins)) >= 8, module
+    for pins in PIN_MODULES:
+        assert sum(1 for _ in _pin_calls(pins)) >= 8, pins.__name__
 
 
 def test_unmutated_oracle_passes_every_pin():
-    for module, (pins, attr) in TARGETS.items():
-        for name, fn, kw in _pin_calls(pins):
-            fn(**kw)
+    for name, fn, kw in _all_pin_calls():
+        fn(**kw)
 
 
 @pytest.mark.parametrize("case", list(MUTATIONS))
 def test_pins_catch_the_mistake(case, monkeypatch):
     module, old, new = MUTATIONS[case]
-    pins, attr = TARGETS[module]
-    monkeypatch.setattr(pins, attr, _mutant(module, old, new))
-    for name, fn, kw in _pin_calls(pins):
+    mutant = _mutant(module, old, new)
+    for user, attr in USES[module]:
+        monkeypatch.setattr(user, attr, mutant)
+    for name, fn, kw in _all_pin_calls():
         try:
             fn(**kw)
         except (Exception, pytest.fail.Exception):  # a failed check, or any error it causes
             return
-    pytest.fail(f"no pin in {pins.__name__} fails with the mistake {case!r}")
+    pytest.fail(f"no pin fails with the mistake {case!r}")
