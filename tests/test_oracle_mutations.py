@@ -48,6 +48,13 @@ MUTATIONS = {
     "grow-middle-lse-of-own-row": ("treegraft_oracle",
                                    "edge[v] = np.float32(row[token[v]] - lse_m[parent[v]])",
                                    "edge[v] = np.float32(row[token[v]] - lse_m[v])"),
+    "bf16-decode-no-shift": ("treegraft_oracle",
+                             "b = np.ascontiguousarray(bits).view(np.uint16).astype(np.uint32) << 16",
+                             "b = np.ascontiguousarray(bits).view(np.uint16).astype(np.uint32)"),
+    "argmax-ties-to-higher-token": ("treegraft_oracle",
+                                    "np.array([int(np.argmax(_row_values(target_logits, r, bf16))) for r in rows],",
+                                    "np.array([len(_row_values(target_logits, r, bf16)) - 1 - int(np.argmax("
+                                    "_row_values(target_logits, r, bf16)[::-1])) for r in rows],"),
     # tree attention
     "attn-scale-1/D": ("treegraft_oracle", "scale = 1.0 / np.sqrt(D)", "scale = 1.0 / D"),
     "attn-gqa-modulo": ("treegraft_oracle", "kv = h // G", "kv = h % Hkv"),
