@@ -50,6 +50,7 @@ def parse():
     p.add_argument("--sets", type=int, default=8)
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-serving", action="store_true", help="skip the batched serving sweep")
     return p.parse_args()
 
 
@@ -224,7 +225,7 @@ def prune_timing(R, seed, dev, stream, reps):
             "in_step": False, "note": "Algorithm 3 on the pre-pruning tree, latency-bound"}
 
 
-EXTRA_CONFIGS = ["llama3-70b-verify", "graft-mha"]
+EXTRA_CONFIGS = ["llama3-70b-verify", "graft-mha", "tiny"]
 
 
 def config_timing(name, seed, dev, stream, n_sets=2, seconds=0.15):
@@ -339,6 +340,245 @@ def config_timing(name, seed, dev, stream, n_sets=2, seconds=0.15):
         out[kname] = ent
     return {"shape": {k_: v_ for k_, v_ in sh.items() if k_ in ("B", "P", "n", "Hq", "Hkv", "D", "V", "k", "N")},
             "kernels": out, "sets": n_sets}
+
+
+SERVING_BATCHES = [1, 2, 4, 8, 16, 32, 64]
+
+
+def _attn_costs(parent, node_off, prefix_len, Hq, Hkv, D):
+    """Algorithmic bytes (K/V of prefix and tree, q and o) and FLOPs
+    (4 Hq D per visible key of every node) of one tree_attn launch."""
+    kv_bytes, keys = 0, 0
+    n_total = int(node_off[-1])
+    for b in range(len(node_off) - 1):
+        lo, hi = int(node_off[b]), int(node_off[b + 1])
+        P = int(prefix_len[b])
+        depth = [0] * (hi - lo)
+        for v in range(1, hi - lo):
+            depth[v] = depth[int(parent[lo + v])] + 1
+        keys += sum(P + d + 1 for d in depth)
+        kv_bytes += 2 * (P + hi - lo) * Hkv * D * 2
+    return kv_bytes + 2 * n_total * Hq * D * 2, 4 * Hq * D * keys
+
+
+def serving_timing(B, dev, stream, seconds=0.12):
+    """One point of the batched serving sweep: B trees with prefixes
+    log-uniform in [512, 32768], 32-256 nodes, depth 4-10 (synth's serving
+    shape, seed 1000 + B), GQA 32/8, head_dim 128, Llama-3 vocabulary, top-10.
+    q/k/v ~ N(0, 1) and the drafter and target logits ~ N(0, 3^2) are drawn
+    on the device from a generator seeded 1000 + B and rounded to bf16; the
+    stronger drafter's fp32 rows likewise.  Per kernel: launch time over
+    rotating input sets (enough that a cycle touches more than the L2), GB/s
+    and, for the attention, TFLOP/s and the roofline fraction.  A step is
+    tree_attn -> expand_topk -> rescore_select -> accept on one input set."""
+    import numpy as np
+    import torch
+    import paper_2608_26112_gb300 as tg
+    from paper_2608_26112_gb300 import synth
+
+    shape = synth.serving_shape(B, seed=0)
+    rng = synth.make_rng(1000 + B)
+    parent, token, node_off = synth.make_trees(rng, shape)
+    Hq, Hkv, D, V, k, N = 32, 8, 128, synth.LLAMA3_VOCAB, 10, 10
+    P = np.asarray(shape["P"], np.int32)
+    ns = np.diff(node_off)
+    n_total, mx = int(node_off[-1]), int(ns.max())
+    S_max = int((P + ns).max())
+    set_bytes = (2 * B * Hkv * S_max * D * 2 + 2 * n_total * V * 2 + n_total * V * 4)
+    R = int(min(4, max(1, -(-400 * 2 ** 20 // set_bytes))))
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1000 + B)
+
+    def randn_bf16(shape_, sigma=1.0, rows_per=512):
+        out = torch.empty(shape_, dtype=torch.bfloat16, device=dev)
+        flat = out.view(shape_[0], -1)
+        for r0 in range(0, shape_[0], rows_per):
+            r1 = min(shape_[0], r0 + rows_per)
+            flat[r0:r1] = torch.randn((r1 - r0, flat.shape[1]), generator=gen, device=dev).mul_(sigma)
+        return out
+
+    t32 = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    vis = np.zeros(n_total, np.uint8)
+    sets = []
+    for _ in range(R):
+        kv = [randn_bf16((B * Hkv, S_max, D), rows_per=8).view(B, Hkv, S_max, D) for _ in range(2)]
+        strong = torch.empty(n_total, V, dtype=torch.float32, device=dev)
+        for r0 in range(0, n_total, 512):
+            r1 = min(n_total, r0 + 512)
+            strong[r0:r1] = torch.randn((r1 - r0, V), generator=gen, device=dev).mul_(3.0).sub_(
+                float(np.log(V)) + 4.5).clamp_(max=0.0)
+        d = dict(q=randn_bf16((n_total, Hq, D)), k=kv[0], v=kv[1], prefix_len=t32(P),
+                 parent=t32(parent), token=t32(token), node_off=t32(node_off),
+                 logits=randn_bf16((n_total, V), 3.0), target=randn_bf16((n_total, V), 3.0),
+                 parent_score=torch.zeros(n_total, device=dev),
+                 weak_edge=torch.full((n_total,), -12.0, device=dev), visited=t32(vis),
+                 strong=strong)
+        o = dict(o=torch.empty_like(d["q"]),
+                 tok=torch.empty(n_total, k, dtype=torch.int32, device=dev),
+                 lp=torch.empty(n_total, k, dtype=torch.float32, device=dev),
+                 sc=torch.empty(n_total, k, dtype=torch.float32, device=dev),
+                 edge=torch.empty(n_total, dtype=torch.float32, device=dev),
+                 score=torch.empty(n_total, dtype=torch.float32, device=dev),
+                 sel=torch.empty(B, N, dtype=torch.int32, device=dev),
+                 nsel=torch.empty(B, dtype=torch.int32, device=dev),
+                 path=torch.empty(B, mx, dtype=torch.int32, device=dev),
+                 alen=torch.empty(B, dtype=torch.int32, device=dev),
+                 bonus=torch.empty(B, dtype=torch.int32, device=dev),
+                 ws=tg.accept_workspace(B, n_total, dev),
+                 attn_ws=torch.zeros(max(16, tg.tree_attn_workspace_size(B, mx, Hq, Hkv, D)),
+                                     dtype=torch.uint8, device=dev))
+        sets.append((d, o))
+
+    def run(kname, d, o):
+        if kname == "tree_attn":
+            tg.tree_attn(d["q"], d["k"], d["v"], d["prefix_len"], d["parent"], d["node_off"], mx,
+                         out=o["o"], ws=o["attn_ws"], stream=stream)
+        elif kname == "expand_topk":
+            tg.expand_topk(d["logits"], d["parent_score"], k, out=(o["tok"], o["lp"], o["sc"]),
+                           stream=stream)
+        elif kname == "rescore_select":
+            tg.rescore_select(d["weak_edge"], d["strong"], d["parent"], d["token"], d["visited"],
+                              d["node_off"], mx, N, out=(o["edge"], o["score"], o["sel"], o["nsel"]),
+                              stream=stream)
+        else:
+            tg.accept(d["target"], d["token"], d["parent"], d["node_off"], mx, mx, o["ws"],
+                      out=(o["path"], o["alen"], o["bonus"]), stream=stream)
+
+    with torch.cuda.stream(stream):
+        for d, o in sets:
+            for kname in KERNELS:
+                run(kname, d, o)
+    stream.synchronize()
+    assert tg.last_device_status(stream) == 0
+    pk, _ = peaks()
+    ab, af = _attn_costs(parent, node_off, P, Hq, Hkv, D)
+    costs = dict(tree_attn=(ab, af), expand_topk=(n_total * V * 2, 0), accept=(n_total * V * 2, 0),
+                 rescore_select=(n_total * 17, 0))
+
+    def timed(fn):
+        g = capture(lambda: [fn(d, o) for d, o in sets], stream)
+        g.replay()
+        t1 = time_graph(g, 2, stream) / (2 * R)
+        reps = max(3, min(2000, int(seconds / max(t1 * R, 1e-7))))
+        return time_graph(g, reps, stream) / (reps * R)
+
+    out = {}
+    for kname in KERNELS:
+        tk = timed(lambda d, o, kname=kname: run(kname, d, o))
+        b_, f_ = costs[kname]
+        ent = {"us": tk * 1e6, "bytes": b_, "GBps": b_ / tk / 1e9,
+               "hbm_frac": b_ / tk / 1e9 / pk["hbm_gbs"]}
+        if f_:
+            roof = max(b_ / (pk["hbm_gbs"] * 1e9), f_ / (pk["bf16_tflops"] * 1e12))
+            ent.update(TFLOPs=f_ / tk / 1e12, tensor_frac=f_ / tk / 1e12 / pk["bf16_tflops"],
+                       roofline_frac=roof / tk,
+                       bound="tensor" if f_ / (pk["bf16_tflops"] * 1e12) > b_ / (pk["hbm_gbs"] * 1e9)
+                       else "hbm")
+        out[kname] = ent
+    t_step = timed(lambda d, o: [run(kn, d, o) for kn in KERNELS])
+    res = {"B": B, "prefix_min": int(P.min()), "prefix_max": int(P.max()),
+           "prefix_mean": float(P.mean()), "nodes": int(n_total), "nodes_max": mx,
+           "sets": R, "kernels": out, "step_us": t_step * 1e6, "steps_per_s": 1.0 / t_step,
+           "launches_per_step": len(KERNELS)}
+    del sets
+    torch.cuda.empty_cache()
+    return res
+
+
+def graft_pipeline_timing(seed, dev, stream, seconds=0.15, n_sets=4):
+    """The two-drafter grafting step of the MHA drafter shape as one
+    CUDA-graph step: the drafter's tree attention over its 64-node tree
+    (32 heads, head_dim 128, prefix 1024), rescoring of all 64 nodes from the
+    stronger drafter's fp32 log-probs (32000 tokens; weak log-probs +
+    N(0, 0.5^2)), reselection of the top 16 grafting positions, expansion of
+    each by its top-8 tokens with the children grafted onto the tree (192
+    nodes), then greedy acceptance on bf16 target logits of the grafted
+    tree.  n_sets rotating input sets; per-kernel launch times beside."""
+    import numpy as np
+    import torch
+    import paper_2608_26112_gb300 as tg
+    from paper_2608_26112_gb300 import synth
+
+    n, V, N, k = 64, 32000, 16, 8
+    cap = n + N * k
+    sets = []
+    for r in range(n_sets):
+        wl = synth.make_workload("graft-mha", seed=seed + r, with_logits=False, with_strong=False)
+        sh = wl["shape"]
+        rng = synth.make_rng(60_000 + seed + r)
+        weak_lp = synth.normal_f32(rng, (n, V), 3.0, -np.log(V) - 4.5)
+        strong_lp = (weak_lp + synth.normal_f32(rng, (n, V), 0.5)).astype(np.float32)
+        weak_edge = np.zeros(n, np.float32)
+        weak_edge[1:] = weak_lp[wl["parent"][1:], wl["token"][1:]]
+        tl = synth.f32_to_bf16_bits(synth.normal_f32(rng, (cap, V), 3.0))
+        bf = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(torch.bfloat16)
+        t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        d = dict(q=bf(wl["q"]), k=bf(wl["k_cache"]), v=bf(wl["v_cache"]),
+                 prefix_len=t(wl["prefix_len"]), node_off=t(wl["node_off"]),
+                 node_off2=torch.tensor([0, cap], dtype=torch.int32, device=dev),
+                 weak_edge=t(weak_edge), strong=t(strong_lp),
+                 visited=torch.zeros(n, dtype=torch.uint8, device=dev),
+                 target=bf(tl), parent0=t(wl["parent"]), token0=t(wl["token"]))
+        o = dict(o=torch.empty_like(d["q"]),
+                 parent=torch.zeros(cap, dtype=torch.int32, device=dev),
+                 token=torch.zeros(cap, dtype=torch.int32, device=dev),
+                 edge=torch.zeros(cap, dtype=torch.float32, device=dev),
+                 score=torch.zeros(cap, dtype=torch.float32, device=dev),
+                 sel=torch.empty(1, N, dtype=torch.int32, device=dev),
+                 nsel=torch.empty(1, dtype=torch.int32, device=dev),
+                 path=torch.empty(1, cap, dtype=torch.int32, device=dev),
+                 alen=torch.empty(1, dtype=torch.int32, device=dev),
+                 bonus=torch.empty(1, dtype=torch.int32, device=dev),
+                 ws=tg.accept_workspace(1, cap, dev),
+                 attn_ws=torch.zeros(max(16, tg.tree_attn_workspace_size(
+                     1, n, sh["Hq"], sh["Hkv"], sh["D"])), dtype=torch.uint8, device=dev))
+        o["parent"][:n] = d["parent0"]
+        o["token"][:n] = d["token0"]
+        sets.append((d, o))
+
+    def stage(name, d, o):
+        if name == "tree_attn":
+            tg.tree_attn(d["q"], d["k"], d["v"], d["prefix_len"], o["parent"][:n], d["node_off"], n,
+                         out=o["o"], ws=o["attn_ws"], stream=stream)
+        elif name == "rescore_select":
+            tg.rescore_select(d["weak_edge"], d["strong"], o["parent"][:n], o["token"][:n],
+                              d["visited"], d["node_off"], n, N,
+                              out=(o["edge"][:n], o["score"][:n], o["sel"], o["nsel"]), stream=stream)
+        elif name == "graft_expand":
+            tg.graft_expand(d["strong"], o["sel"], k, cap, n, o["parent"], o["token"], o["edge"],
+                            o["score"], stream=stream)
+        else:
+            tg.accept(d["target"], o["token"], o["parent"], d["node_off2"], cap, cap, o["ws"],
+                      out=(o["path"], o["alen"], o["bonus"]), stream=stream)
+
+    names = ["tree_attn", "rescore_select", "graft_expand", "accept"]
+    with torch.cuda.stream(stream):
+        for d, o in sets:
+            for nm in names:
+                stage(nm, d, o)
+    stream.synchronize()
+    assert tg.last_device_status(stream) == 0
+
+    def timed(fn):
+        g = capture(lambda: [fn(d, o) for d, o in sets], stream)
+        g.replay()
+        t1 = time_graph(g, 2, stream) / (2 * n_sets)
+        reps = max(3, min(4000, int(seconds / max(t1 * n_sets, 1e-7))))
+        return time_graph(g, reps, stream) / (reps * n_sets)
+
+    t_step = timed(lambda d, o: [stage(nm, d, o) for nm in names])
+    per = {nm: timed(lambda d, o, nm=nm: stage(nm, d, o)) * 1e6 for nm in names}
+    d0 = sets[0][0]
+    ab, af = _attn_costs(sets[0][1]["parent"][:n].cpu().numpy(), [0, n], [1024], 32, 32, 128)
+    bytes_ = {"tree_attn": ab, "rescore_select": n * 17 + 64 * 4,
+              "graft_expand": N * V * 4 + N * k * 16, "accept": cap * V * 2}
+    kern = {nm: {"us": per[nm], "bytes": bytes_[nm], "GBps": bytes_[nm] / per[nm] / 1e3}
+            for nm in names}
+    kern["tree_attn"]["TFLOPs"] = af / per["tree_attn"] / 1e6
+    return {"shape": {"P": 1024, "n": n, "n_grafted": cap, "Hq": 32, "Hkv": 32, "D": 128, "V": V,
+                      "N": N, "k": k},
+            "step_us": t_step * 1e6, "steps_per_s": 1.0 / t_step, "launches_per_step": len(names),
+            "kernels": kern, "sets": n_sets}
 
 
 GROW_SCHEDULE = [1, 0, 1, 0, 1]
@@ -777,6 +1017,9 @@ def ours_arm(args):
         ngram = ngram_timing(rank_seed(args.seed, rank), dev, stream, kreps)
         extra = {nm: config_timing(nm, rank_seed(args.seed, rank), dev, stream)
                  for nm in EXTRA_CONFIGS}
+        extra["graft-mha-pipeline"] = graft_pipeline_timing(rank_seed(args.seed, rank), dev, stream)
+        if not args.no_serving:
+            extra["serving-sweep"] = [serving_timing(B, dev, stream) for B in SERVING_BATCHES]
     assert tg.last_device_status(stream) == 0
     t_max = max_over_ranks(t_steps, world)
     steps_per_s = job_throughput(world, K, t_max)

@@ -20,8 +20,11 @@
  *    rows [node_off[b], node_off[b+1]); inside a tree, parent[] holds LOCAL
  *    ids with parent[0] = -1 and 0 <= parent[i] < i (parents before
  *    children, the order Algorithm 3 re-indexes the verification tree into).
- *    node_off[0] = 0.  Every tree has at least one node (its root) and at
- *    most 256 nodes.
+ *    node_off[0] = 0 and node_off[B] = n_total (the trees cover the node
+ *    rows exactly).  Every tree has at least one node (its root) and at
+ *    most 256 nodes.  node_off lives on the device, so these conditions are
+ *    checked there: a row that falls outside every tree's extent sets
+ *    TG_ERR_DEVICE_TREE and takes no part in any tree's result.
  *  - bf16 data is IEEE bfloat16 (raw 16-bit patterns); all fp32/int32 data
  *    is native-endian.
  */
@@ -80,9 +83,12 @@ typedef enum { TG_BF16 = 0, TG_F32 = 1 } tg_dtype;
  *          Hkv, D) bytes, 16-byte aligned, ZERO-FILLED before its first use:
  *          split counters (returned to zero by every call) and the partial
  *          rows of the split-KV combine.  Calls sharing one ws must not
- *          overlap on the GPU.  When the whole grid fits on the GPU at once
- *          the launch is cooperative and the splits of a work item meet on
- *          those counters (a bounded wait: TG_ERR_TIMEOUT, never a hang).
+ *          overlap on the GPU.  Small problems split the keys of a work
+ *          unit over several thread blocks of a cooperative launch (the
+ *          whole grid resident at once) that meet on those counters (a
+ *          bounded wait, see treegraft_set_wait_budget: TG_ERR_TIMEOUT,
+ *          never a hang).  The size is 0 when these sizes never split; ws
+ *          may then be NULL.
  * Errors: TG_ERR_INVALID_ARG (null pointer, bad sizes, misaligned q/k/v),
  *   TG_ERR_UNSUPPORTED (D or G outside the list), TG_ERR_CUDA.  A malformed
  *   tree sets TG_ERR_DEVICE_TREE; its rows of `out` and `lse_out` are then
@@ -99,6 +105,22 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
  * needs for these sizes (0 for invalid sizes).  Depends on no device state.
  */
 size_t treegraft_tree_attn_workspace_size(int B, int max_nodes, int Hq, int Hkv, int D);
+
+/*
+ * treegraft_set_wait_budget - bound, in SM clock cycles, of the waits a
+ * kernel makes on OTHER thread blocks: the split barrier of
+ * treegraft_tree_attn, whose counters live in the caller's workspace.  A
+ * wait that runs out raises TG_ERR_TIMEOUT in the device status word and
+ * the kernel returns (that call's outputs are then undefined); the
+ * counters are returned to zero, so the next call on the same workspace is
+ * exact.  Waits inside one thread block (copies and tensor-core products)
+ * keep their own fixed bound of about one second.  The budget applies to
+ * the calls launched after it is set, process-wide.  cycles = 0 restores
+ * the default (about one second at the GB300's maximum SM clock).  No
+ * counterpart in the paper: this is a failure-detection control.
+ * Errors: TG_ERR_INVALID_ARG for cycles < 0.
+ */
+int treegraft_set_wait_budget(int64_t cycles);
 
 /*
  * treegraft_expand_topk - per-node log-softmax, top-k children, path scores.
@@ -175,6 +197,42 @@ int treegraft_rescore_select(const float* weak_edge, const float* strong_lp, int
 size_t treegraft_accept_workspace_size(int B, int n_total);
 
 /*
+ * treegraft_graft_expand - expand the reselected grafting positions and
+ * graft their children into the shared tree, non-destructively.
+ *
+ * Paper: the middle-drafter step of Sec. 3.2 / Algorithm 2 - after the
+ * candidate pool is rescored and Top_W reselects grafting positions
+ * (treegraft_rescore_select), each position v gets the drafter's top-m
+ * next tokens as new children, appended to the tree without replacing any
+ * existing node ("non-destructive grafting"), with edge score
+ * p(u) = q(y | pi(v)) and path score s(u) = s(v) p(u) (log domain: sum).
+ *
+ * Trees use a capacity layout: tree b's nodes are rows [b*cap, b*cap + n)
+ * of parent / token / edge / score, and the grafted children go to rows
+ * b*cap + n + i*k + j for position slot i < N and rank j < k (the graft of
+ * slot i is in slot order, its children in rank order).
+ *   v      = selected[b*N + i]         (a LOCAL node id, 0 <= v < n)
+ *   row    = logits row b*cap + v      (the drafter's next-token logits
+ *                                       under the prefix ending at v)
+ *   child j: parent = v, token = j-th largest logit of row (ties to the
+ *            lower token), edge = logit - lse(row),
+ *            score = fp32(score[b*cap + v] + edge)
+ * logits   [logit_rows, ld] elements of dtype; rows must exist for every
+ *          selected node.  V <= 262144 (bf16) / 131072 (fp32).
+ * selected int32 [B, N], as treegraft_rescore_select writes it.  1 <= k <=
+ *          min(V, 32); n + N*k <= cap.
+ * parent, token int32 [B*cap]; edge, score fp32 [B*cap]: read at the
+ *          selected rows, written at the appended rows.
+ * Errors: TG_ERR_INVALID_ARG, TG_ERR_UNSUPPORTED, TG_ERR_CUDA.  A selected
+ *   id outside [0, n), or a logits row past logit_rows, sets
+ *   TG_ERR_DEVICE_INDEX and that slot's children are left unwritten.
+ */
+int treegraft_graft_expand(const void* logits, int dtype, int logit_rows, int V, int64_t ld,
+                           int B, int N, const int32_t* selected, int k, int cap, int n,
+                           int32_t* parent, int32_t* token, float* edge, float* score,
+                           void* stream);
+
+/*
  * treegraft_accept - greedy longest-accepted-path walk (temperature 0).
  *
  * Paper: verification of the pruned tree with the target model and the
@@ -223,6 +281,10 @@ int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld,
  * launch nothing.
  * The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * The address is kept for the life of the process: after cudaDeviceReset
+ * (or anything else that destroys the device's primary context) it is stale,
+ * so this library must not be used across such a reset.  The same holds for
+ * the device status word that every call of this header writes.
  * All calls on a device share the one array: calls that overlap on the GPU
  * (other streams, other host threads) race and give wrong results; order
  * them on one stream.  Each call clears the counters it needs on `stream`

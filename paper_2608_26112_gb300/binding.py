@@ -72,6 +72,9 @@ _SIGNATURES = {
                                   _c_vp, _c_vp, _c_int, _c_int, _c_int, _c_int, _c_int, _c_vp,
                                   _c_vp, _c_vp, _c_vp, _c_vp, _c_vp],
     "treegraft_last_device_status": [_c_vp],
+    "treegraft_set_wait_budget": [_c_i64],
+    "treegraft_graft_expand": [_c_vp, _c_int, _c_int, _c_int, _c_i64, _c_int, _c_int, _c_vp,
+                               _c_int, _c_int, _c_int, _c_vp, _c_vp, _c_vp, _c_vp, _c_vp],
     "treegraft_status_string": [_c_int],
 }
 _RESTYPES = {"treegraft_accept_workspace_size": _c_size,
@@ -326,6 +329,39 @@ def accept_noalloc(target_logits, token, parent, node_off, max_nodes, path_cap, 
                                         _ptr(alen), _ptr(bonus), _stream(stream))
     _check("treegraft_accept_noalloc", st)
     return path, alen, bonus
+
+
+def graft_expand(logits, selected, k, cap, n, parent, token, edge, score, *, V=None,
+                 stream=None):
+    """Expand the reselected grafting positions (selected [B, N] int32, local
+    node ids) by their top-k tokens from the drafter's rows (logits row
+    b * cap + v) and append the children to the capacity-layout tree arrays
+    parent / token / edge / score [B * cap] at rows b * cap + n + i * k + j.
+    In place; returns (parent, token, edge, score)."""
+    _need(selected, torch.int32, "selected")
+    for t, nm, dt in ((parent, "parent", torch.int32), (token, "token", torch.int32),
+                      (edge, "edge", torch.float32), (score, "score", torch.float32)):
+        _need(t, dt, nm)
+    if logits.dim() != 2:
+        raise ValueError("logits must be [rows, ld]")
+    if not logits.is_cuda or logits.stride(1) != 1:
+        raise ValueError("logits must be a CUDA tensor with unit element stride")
+    B, N = selected.shape
+    if parent.numel() < B * cap:
+        raise ValueError("tree arrays hold fewer than B * cap nodes")
+    V = logits.shape[1] if V is None else int(V)
+    st = lib().treegraft_graft_expand(_ptr(logits), _logit_dtype(logits), logits.shape[0], V,
+                                      logits.stride(0), B, N, _ptr(selected), int(k), int(cap),
+                                      int(n), _ptr(parent), _ptr(token), _ptr(edge), _ptr(score),
+                                      _stream(stream))
+    _check("treegraft_graft_expand", st)
+    return parent, token, edge, score
+
+
+def set_wait_budget(cycles: int) -> None:
+    """Bound (SM cycles) of the waits a kernel makes on other thread blocks
+    (the split barrier of tree_attn); 0 restores the default."""
+    _check("treegraft_set_wait_budget", lib().treegraft_set_wait_budget(int(cycles)))
 
 
 def last_device_status(stream=None) -> int:

@@ -97,7 +97,11 @@ __global__ void __launch_bounds__(kScanThreads, 4) accept_kernel(AcceptArgs a, i
   if (crank != 0) return;
 
   // leader: publish the argmax, take a ticket for the row's tree
-  const bool bad_tree = (n < 1 || n > 256 || off < 0 || off + n > a.n_total);
+  // a row outside its tree's own extent (node_off[0] > 0 or node_off[B] <
+  // n_total) belongs to no tree: it must not draw a ticket of the tree the
+  // search landed on, or that tree's walk could run before its own rows
+  const bool bad_tree = (n < 1 || n > 256 || off < 0 || off + n > a.n_total || row < off ||
+                         row >= off + n);
   if (tid == 0) {
     uint64_t best = 0;
     for (int c = 0; c < C; ++c) best = sm.recv_key[c] > best ? sm.recv_key[c] : best;

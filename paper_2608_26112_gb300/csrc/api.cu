@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <mutex>
@@ -24,6 +25,8 @@ constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 int* g_status_ptr[kMaxDevices] = {};
 int g_sm_count[kMaxDevices] = {};
+// bound of the waits on other CTAs (treegraft_set_wait_budget)
+std::atomic<long long> g_wait_budget{kInterBlockWaitCycles};
 
 int current_device() {
   int d = 0;
@@ -125,8 +128,13 @@ extern "C" {
 
 size_t treegraft_tree_attn_workspace_size(int B, int max_nodes, int Hq, int Hkv, int D) {
   if (B < 1 || max_nodes < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || (D != 64 && D != 128)) return 0;
-  const int mtiles = ((Hq / Hkv) * max_nodes + 127) / 128;
-  return tree_attn_ws_bytes(D, B, Hkv, mtiles, kAttnMaxSplits);
+  return tree_attn_ws_bytes(D, B, Hkv, Hq / Hkv, max_nodes);
+}
+
+int treegraft_set_wait_budget(int64_t cycles) {
+  if (cycles < 0) return TG_ERR_INVALID_ARG;
+  g_wait_budget.store(cycles > 0 ? (long long)cycles : kInterBlockWaitCycles);
+  return TG_OK;
 }
 
 int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
@@ -181,12 +189,16 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
   a.out = out;
   a.lse_out = lse_out;
   a.status = st;
-  const int mtiles = (G * max_nodes + 127) / 128;
-  const AttnPlan plan = tree_attn_plan(D, B, Hkv, mtiles, S_max, device_sm_count());
-  const size_t need = tree_attn_ws_bytes(D, B, Hkv, mtiles, plan.splits);
-  if (need > 0 && (ws == nullptr || ws_bytes < need || !aligned16(ws))) return TG_ERR_INVALID_ARG;
+  const AttnPlan plan = tree_attn_plan(D, B, Hkv, G, max_nodes, S_max, device_sm_count());
+  a.unit_rows = plan.unit_rows;
+  a.rblocks = tree_attn_rblocks(G, max_nodes, plan.unit_rows);
+  if (plan.splits > 1) {
+    const size_t need = tree_attn_ws_bytes(D, B, Hkv, G, max_nodes);
+    if (ws == nullptr || ws_bytes < need || !aligned16(ws)) return TG_ERR_INVALID_ARG;
+  }
   a.ws = ws;
-  a.coop = plan.coop;
+  a.lpt = plan.lpt;
+  a.split_wait_cycles = g_wait_budget.load();
   return launch_tree_attn(tq, tk, tv, a, plan, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? TG_OK
              : TG_ERR_CUDA;
@@ -347,6 +359,46 @@ int treegraft_grow_step(int mode, const void* logits, int dtype, int V, int64_t 
   a.status = st;
   grow_ws_carve(a, ws, B, cap, m);
   return launch_grow_step(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK : TG_ERR_CUDA;
+}
+
+int treegraft_graft_expand(const void* logits, int dtype, int logit_rows, int V, int64_t ld,
+                           int B, int N, const int32_t* selected, int k, int cap, int n,
+                           int32_t* parent, int32_t* token, float* edge, float* score,
+                           void* stream) {
+  if (!logits || !selected || !parent || !token || !edge || !score) return TG_ERR_INVALID_ARG;
+  if (dtype != TG_BF16 && dtype != TG_F32) return TG_ERR_INVALID_ARG;
+  if (B < 1 || N < 1 || k < 1 || k > V || V < 1 || ld < V || logit_rows < 1 || n < 1 ||
+      cap < 1 || (long long)n + (long long)N * k > (long long)cap)
+    return TG_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(logits) & (dtype == TG_BF16 ? 1 : 3)) != 0)
+    return TG_ERR_INVALID_ARG;  // elements must sit at their natural alignment
+  if (k > TG_MAX_TOPK || V > (dtype == TG_BF16 ? 262144 : 131072) ||
+      (long long)B * cap > (1ll << 30) || (long long)B * N > (1ll << 30))
+    return TG_ERR_UNSUPPORTED;
+  int* st = status_ptr();
+  if (!st) return TG_ERR_CUDA;
+  TopkArgs a = {};
+  a.logits = logits;
+  a.is_bf16 = dtype == TG_BF16;
+  a.logit_rows = logit_rows;
+  a.V = V;
+  a.ld = ld;
+  a.rows = B * N;
+  a.row_idx = selected;
+  a.idx_local = 1;
+  a.parent_score = score;
+  a.ps_gather = 1;
+  a.k = k;
+  a.gdiv = N;
+  a.gcap = cap;
+  a.app_n = n;
+  a.app_parent = parent;
+  a.app_token = token;
+  a.app_edge = edge;
+  a.app_score = score;
+  a.status = st;
+  return launch_expand_topk(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TG_OK
+                                                                               : TG_ERR_CUDA;
 }
 
 int treegraft_accept(const void* target_logits, int dtype, int V, int64_t ld, const int32_t* token,

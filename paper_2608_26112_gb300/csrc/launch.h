@@ -13,27 +13,36 @@ struct AttnArgs {
   const int32_t* parent;
   const int32_t* node_off;
   int B, max_nodes, n_total, Hq, Hkv, D, S_max;
+  int unit_rows;     // query rows per work unit: 256 (two tiles) or 128 (one)
+  int rblocks;       // units per (tree, kv-head) at max_nodes
   float scale_log2;  // softmax scale * log2(e)
   void* out;
   float* lse_out;
   void* ws;  // split counters + combine partial rows (tree_attn_ws_bytes)
   int* status;
-  int coop;  // 1: cooperative launch, split barrier on counters in ws; 0: clusters
+  int lpt;   // 1: one CTA per unit, units dealt longest tree first (1-D grid)
+  long long split_wait_cycles;  // bound of the wait on the other splits of a unit
 };
-// How one launch splits the keys: `splits` CTAs per work item, joined by a
-// thread-block cluster or, with coop, by a cooperative launch whose whole
-// grid is resident at once.
+// How one launch cuts the work: `splits` CTAs per unit (the key tiles dealt
+// round-robin; > 1 needs a cooperative launch whose whole grid is resident
+// at once), and whether units are dealt longest tree first.
 struct AttnPlan {
   int splits;
-  int coop;
+  int lpt;
+  int unit_rows;
 };
+constexpr int kAttnMaxSplits = 32;
+// default bound of the waits on other thread blocks: about one second at the
+// GB300's maximum SM clock (the same bound as the in-block mbarrier waits)
+constexpr long long kInterBlockWaitCycles = 2000000000LL;
+constexpr int kAttnMaxCoopCtas = 256;  // split plans never exceed this many CTAs
 // tmaps: q [D, Hq, n_total], k and v [D, B*Hkv*S_max] (innermost first)
 cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                              const CUtensorMap& tm_v, const AttnArgs& a, AttnPlan plan,
                              cudaStream_t s);
-AttnPlan tree_attn_plan(int D, int B, int Hkv, int mtiles, int S_max, int num_sms);
-size_t tree_attn_ws_bytes(int D, int B, int Hkv, int mtiles, int splits);
-constexpr int kAttnMaxSplits = 10;
+int tree_attn_rblocks(int G, int max_nodes, int unit_rows);
+AttnPlan tree_attn_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max, int num_sms);
+size_t tree_attn_ws_bytes(int D, int B, int Hkv, int G, int max_nodes);
 
 struct TopkArgs {
   const void* logits;
@@ -61,6 +70,10 @@ struct TopkArgs {
   float* app_edge;
   float* app_score;
   int row0;  // first logical row of this launch (grids of at most 65535 rows)
+  // Graft (with app_token and row_idx): row_idx holds LOCAL node ids of
+  // tree i / gdiv (read at (i / gdiv) * gcap + id, id < app_n), and with
+  // ps_gather the parent score is parent_score[that physical row].
+  int idx_local, ps_gather;
 };
 cudaError_t launch_expand_topk(const TopkArgs& a, cudaStream_t s);
 int scan_cluster_size(int V, int is_bf16, int rows, int num_sms);

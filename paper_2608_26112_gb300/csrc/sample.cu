@@ -130,7 +130,9 @@ __global__ void __launch_bounds__(kScanThreads, 4) sample_kernel(SampleArgs a, i
   }
   const int off = __ldg(a.node_off + b);
   const int n = __ldg(a.node_off + b + 1) - off;
-  const bool bad_tree = (n < 1 || n > 256 || off < 0 || off + n > a.n_total);
+  // a row outside its tree's own extent belongs to no tree and draws no ticket
+  const bool bad_tree = (n < 1 || n > 256 || off < 0 || off + n > a.n_total || row < off ||
+                         row >= off + n);
   int v_par = -1, v_tok = 0;
   if (!bad_tree && tid < n) {
     v_par = __ldg(a.parent + off + tid);

@@ -230,6 +230,10 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   int r = row;
   if (a.row_idx) {
     r = a.row_idx[row];
+    if (kTree && a.idx_local) {  // a local node id of tree row / gdiv (graft)
+      const int bt = row / a.gdiv;
+      r = (r >= 0 && r < a.app_n) ? bt * a.gcap + r : -1;
+    }
   } else if (kTree && a.gdiv) {
     const int bt = row / a.gdiv;
     r = bt * a.gcap + a.goff + (row - bt * a.gdiv);
@@ -244,7 +248,8 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   // the leader's threads fetch the parent's path score now, while the
   // logits are in flight (one broadcast request per warp)
   float parent_score = 0.f;
-  if (crank == 0 && a.parent_score) parent_score = __ldg(a.parent_score + row);
+  if (crank == 0 && a.parent_score)
+    parent_score = __ldg(a.parent_score + ((kTree && a.ps_gather) ? r : row));
   const int per = ((V + C - 1) / C + VW - 1) / VW * VW;
   const int c0 = min(V, crank * per);
   const int c1 = min(V, c0 + per);

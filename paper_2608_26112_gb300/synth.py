@@ -23,7 +23,9 @@ Conventions shared by every array produced here:
 """
 from __future__ import annotations
 
+import json
 import math
+import os
 
 import numpy as np
 
@@ -232,8 +234,11 @@ WORKLOADS = {
     # name: shape parameters (the synthetic stand-ins described in the module doc)
     "tiny": dict(B=1, P=128, n=16, depth=4, cap=None, rank_bias=0.0, Hq=8, Hkv=8,
                  D=64, V=1024, logit_dtype="f32", k=4, N=8),
+    # the tree is one of the stored trees grown by Algorithm 1 + GlobalPrune
+    # (tests/golden/llama3_8b_grown_trees.json), chosen by the seed
     "llama3-8b-verify": dict(B=1, P=2048, n=60, depth=6, cap=10, rank_bias=0.35, Hq=32,
-                             Hkv=8, D=128, V=LLAMA3_VOCAB, logit_dtype="bf16", k=10, N=10),
+                             Hkv=8, D=128, V=LLAMA3_VOCAB, logit_dtype="bf16", k=10, N=10,
+                             tree="grown"),
     "graft-mha": dict(B=1, P=1024, n=64, depth=7, cap=8, rank_bias=0.35, Hq=32, Hkv=32,
                       D=128, V=32000, logit_dtype="f32", k=8, N=16),
     "llama3-70b-verify": dict(B=4, P=8192, n=128, depth=8, cap=16, rank_bias=0.25, Hq=64,
@@ -257,13 +262,39 @@ def _as_list(x, B):
     return list(x) if isinstance(x, (list, tuple)) else [x] * B
 
 
-def make_trees(rng, shape: dict):
-    """Concatenated trees of a workload: (parent, token, node_off, depth_cap)."""
+GROWN_TREES = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "tests",
+                           "golden", "llama3_8b_grown_trees.json")
+_grown_cache: list = []
+
+
+def grown_trees() -> list:
+    """The stored draft trees of the Llama-3-8B-shaped verify workload: each
+    grown by Algorithm 1 (6 top-10 expansion steps by cumulative
+    log-probability) and pruned to 60 nodes by GlobalPrune, written by
+    tests/golden/make_grown_trees.py.  Loaded, not computed, here."""
+    if not _grown_cache:
+        with open(GROWN_TREES) as f:
+            _grown_cache.extend(json.load(f)["trees"])
+    return _grown_cache
+
+
+def make_trees(rng, shape: dict, seed: int = 0):
+    """Concatenated trees of a workload: (parent, token, node_off).  With
+    shape["tree"] == "grown", tree b is stored tree (seed + b) mod count."""
     B = shape["B"]
     ns = _as_list(shape["n"], B)
     depths = _as_list(shape["depth"], B)
     parents, tokens, off = [], [], [0]
     for b in range(B):
+        if shape.get("tree") == "grown":
+            t = grown_trees()[(seed + b) % len(grown_trees())]
+            p, tk = np.asarray(t["parent"], np.int32), np.asarray(t["token"], np.int32)
+            if len(p) != ns[b]:
+                raise ValueError("stored grown tree has the wrong size")
+            parents.append(p)
+            tokens.append(tk)
+            off.append(off[-1] + ns[b])
+            continue
         p = sample_tree(rng, ns[b], depths[b], shape.get("cap"), shape.get("rank_bias", 0.0))
         parents.append(p)
         tokens.append(sample_tokens(rng, ns[b], shape["V"]))
@@ -296,7 +327,7 @@ def make_workload(name_or_shape, seed: int = 0, *, kv_tail: str = "zero",
     shape = dict(WORKLOADS[name_or_shape]) if isinstance(name_or_shape, str) else dict(name_or_shape)
     rng = make_rng(seed)
     B = shape["B"]
-    parent, token, node_off = make_trees(rng, shape)
+    parent, token, node_off = make_trees(rng, shape, seed)
     n_total = int(node_off[-1])
     Ps = _as_list(shape["P"], B)
     ns = [int(node_off[b + 1] - node_off[b]) for b in range(B)]

@@ -132,6 +132,42 @@ def test_tree_attn_malformed_tree_sets_status(dev):
     assert tg.last_device_status() == 0                  # cleared by the read
 
 
+def test_tree_attn_split_wait_runs_out_and_recovers(dev):
+    """The split barrier of tree_attn is a bounded wait on other thread
+    blocks, on counters in the caller's workspace.  A workspace whose first
+    counter holds a value the splits can never bring up to their count (as a
+    corrupted workspace would) makes every split of that unit give up after
+    a short budget: the call returns, TG_ERR_TIMEOUT is set, the unit's two
+    counters are back at zero and the next call on the same workspace is
+    exact.  Nothing waits without a bound, so no GPU hang is involved."""
+    wl = synth.make_workload("llama3-8b-verify", seed=5, with_logits=False, with_strong=False)
+    sh = wl["shape"]
+    q = _dev.bf16(wl["q"], dev)
+    k, v = _dev.bf16(wl["k_cache"], dev), _dev.bf16(wl["v_cache"], dev)
+    pl, par, off = (_dev.i32(wl["prefix_len"], dev), _dev.i32(wl["parent"], dev),
+                    _dev.i32(wl["node_off"], dev))
+    n = len(wl["parent"])
+    nbytes = tg.tree_attn_workspace_size(1, n, sh["Hq"], sh["Hkv"], sh["D"])
+    assert nbytes > 0                                    # this shape runs a split plan
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+    ws.view(torch.int32)[0] = -1000                      # unit 0's arrival counter
+    tg.set_wait_budget(20_000)                           # ~10 us at the GB300's clock
+    try:
+        tg.tree_attn(q, k, v, pl, par, off, n, ws=ws)
+        torch.cuda.synchronize()
+        st = tg.last_device_status()
+    finally:
+        tg.set_wait_budget(0)
+    assert st & 8, st                                    # TG_ERR_TIMEOUT
+    assert ws.view(torch.int32)[:2].tolist() == [0, 0]   # counters returned to zero
+    lse = torch.empty(n, sh["Hq"], device=dev)
+    o, _ = tg.tree_attn(q, k, v, pl, par, off, n, ws=ws, lse_out=lse)
+    _status_clean()
+    ref_o, ref_lse = O.tree_attention(wl["q"], wl["k_cache"], wl["v_cache"], wl["prefix_len"],
+                                      wl["parent"], wl["node_off"], Hkv=sh["Hkv"])
+    _check_attn(wl, _dev.bf16_to_np(o), lse.cpu().numpy().astype(np.float64), ref_o, ref_lse)
+
+
 # ------------------------------------------------------------------ expand_topk
 
 def _run_expand(lg_dev, ps, k, dev, row_idx=None, V=None):
@@ -317,6 +353,33 @@ def test_accept_path_cap_too_small_sets_status(dev):
     assert A[0] == n - 1 and list(path[0]) == list(range(n))
 
 
+@pytest.mark.parametrize("where", ["short-end", "late-start"])
+def test_accept_rows_outside_every_tree_set_status(dev, where):
+    """node_off that does not cover [0, n_total): the uncovered rows belong to
+    no tree, raise TG_ERR_DEVICE_TREE and draw no ticket, so the workspace
+    counters stay clean and the next well-formed call is exact."""
+    wl = synth.make_workload("llama3-70b-verify", seed=21,
+                             with_strong=False)
+    off = wl["node_off"].copy()
+    bad = off.copy()
+    if where == "short-end":
+        bad[-1] -= 3          # the last three rows are in no tree
+    else:
+        bad[0] = 2            # rows 0 and 1 are in no tree
+    lg = _dev.logits(wl, dev)
+    B, n_total = len(off) - 1, len(wl["parent"])
+    ws = tg.accept_workspace(B, n_total, dev)
+    tok, par = _dev.i32(wl["token"], dev), _dev.i32(wl["parent"], dev)
+    cap = _dev.max_nodes(wl)
+    tg.accept(lg, tok, par, _dev.i32(bad, dev), cap, cap, ws)
+    assert tg.last_device_status() & 4
+    got = tg.accept(lg, tok, par, _dev.i32(off, dev), cap, cap, ws)
+    _status_clean()
+    ref = O.accept(wl["logits"], wl["token"], wl["parent"], off, cap, bf16=True)
+    for g, r in zip(got, ref):
+        np.testing.assert_array_equal(g.cpu().numpy(), r)
+
+
 def test_accept_grafting_examples(dev):
     import json, os
     with open(os.path.join(os.path.dirname(__file__), "golden", "grafting_examples.json")) as f:
@@ -378,6 +441,75 @@ def test_graft_step_pipeline(dev):
     rp, rA, rb = O.accept(tl_bits, token, parent, g["node_off"], n2, bf16=True)
     np.testing.assert_array_equal(path, rp)
     assert A[0] == rA[0] and bonus[0] == rb[0]
+
+
+def test_graft_expand_on_device(dev):
+    """The same two-drafter step with the graft on the device
+    (treegraft_graft_expand, capacity layout): rescore + reselect, then the
+    16 selected positions expanded by top-8 from the stronger drafter's rows
+    and their children appended at rows 64.. of the 192-node tree.  Tokens
+    and parents bit-exact, edge and path scores within 1e-4 relative of the
+    oracle's expand_topk of the same rows; then accept on the grafted
+    device arrays equals the oracle's accept."""
+    wl = synth.make_workload("graft-mha", seed=4, with_logits=False, with_strong=False)
+    rng = synth.make_rng(321)
+    n, V, N, k, cap = 64, 32000, 16, 8, 192
+    weak_lp = synth.normal_f32(rng, (n, V), 3.0, -np.log(V) - 4.5)
+    strong_lp = (weak_lp + synth.normal_f32(rng, (n, V), 0.5)).astype(np.float32)
+    weak_edge = np.zeros(n, np.float32)
+    for v in range(1, n):
+        weak_edge[v] = weak_lp[wl["parent"][v], wl["token"][v]]
+    visited = (np.arange(n) < 5).astype(np.uint8)
+    par = torch.full((cap,), -7, dtype=torch.int32, device=dev)
+    tok = torch.full((cap,), -7, dtype=torch.int32, device=dev)
+    edge = torch.zeros(cap, dtype=torch.float32, device=dev)
+    score = torch.zeros(cap, dtype=torch.float32, device=dev)
+    par[:n] = _dev.i32(wl["parent"], dev)
+    tok[:n] = _dev.i32(wl["token"], dev)
+    sel = torch.empty(1, N, dtype=torch.int32, device=dev)
+    nsel = torch.empty(1, dtype=torch.int32, device=dev)
+    strong = _dev.f32(strong_lp, dev)
+    tg.rescore_select(_dev.f32(weak_edge, dev), strong, par[:n], tok[:n], _dev.u8(visited, dev),
+                      _dev.i32(wl["node_off"], dev), n, N,
+                      out=(edge[:n], score[:n], sel, nsel))
+    tg.graft_expand(strong, sel, k, cap, n, par, tok, edge, score)
+    _status_clean()
+    e_o, s_o, sel_o, ns_o = O.rescore_select(weak_edge, strong_lp, wl["parent"], wl["token"],
+                                             visited, wl["node_off"], N)
+    assert int(nsel[0]) == N and int(ns_o[0]) == N
+    np.testing.assert_array_equal(sel.cpu().numpy(), sel_o)
+    tok_o, lp_o, sc_o, _ = O.expand_topk(strong_lp, s_o[sel_o[0]], k, row_idx=sel_o[0])
+    np.testing.assert_array_equal(par.cpu().numpy()[n:], np.repeat(sel_o[0], k))
+    np.testing.assert_array_equal(tok.cpu().numpy()[n:], tok_o.reshape(-1))
+    np.testing.assert_allclose(edge.cpu().numpy()[n:], lp_o.reshape(-1), rtol=SCORE_RTOL, atol=1e-5)
+    np.testing.assert_allclose(score.cpu().numpy()[n:], sc_o.reshape(-1), rtol=SCORE_RTOL, atol=1e-5)
+    np.testing.assert_array_equal(score.cpu().numpy()[:n], s_o)
+    # accept on the grafted device tree
+    parent_h = np.concatenate([wl["parent"], np.repeat(sel_o[0], k)]).astype(np.int32)
+    token_h = np.concatenate([wl["token"], tok_o.reshape(-1)]).astype(np.int32)
+    tl = synth.normal_f32(rng, (cap, V), 3.0)
+    synth.plant_child_bump(rng, tl, parent_h, token_h, np.arange(cap), prob=0.9, bump=40.0)
+    tl_bits = synth.f32_to_bf16_bits(tl)
+    ws = tg.accept_workspace(1, cap, dev)
+    path, A, bonus = tg.accept(_dev.bf16(tl_bits, dev), tok, par,
+                               torch.tensor([0, cap], dtype=torch.int32, device=dev), cap, cap, ws)
+    _status_clean()
+    rp, rA, rb = O.accept(tl_bits, token_h, parent_h, np.array([0, cap], np.int32), cap, bf16=True)
+    np.testing.assert_array_equal(path.cpu().numpy(), rp)
+    assert int(A[0]) == int(rA[0]) and int(bonus[0]) == int(rb[0])
+
+
+def test_graft_expand_bad_selected_sets_status(dev):
+    n, V, N, k, cap = 8, 64, 2, 2, 16
+    lg = torch.zeros(n, V, device=dev)
+    sel = torch.tensor([[3, 9]], dtype=torch.int32, device=dev)   # 9 is not a node
+    par = torch.zeros(cap, dtype=torch.int32, device=dev)
+    tok = torch.zeros(cap, dtype=torch.int32, device=dev)
+    edge = torch.zeros(cap, device=dev)
+    score = torch.zeros(cap, device=dev)
+    tg.graft_expand(lg, sel, k, cap, n, par, tok, edge, score)
+    assert tg.last_device_status() & 16
+    assert par.cpu().numpy()[n:n + k].tolist() == [3, 3]            # the valid slot is grafted
 
 
 # ------------------------------------------------------------------ serving sweep

@@ -66,6 +66,38 @@ def test_accept_noalloc_matches_accept_twice():
         assert tg.last_device_status() == 0
         for g, r in zip(got, ref):
             assert torch.equal(g, r)        # integer outputs: exact
+        # and directly against the CPU oracle
+        from oracle import treegraft_oracle as O
+        from paper_2608_26112_gb300 import synth
+        wl = synth.make_workload(name, seed=seed, with_strong=False)
+        want = O.accept(wl["logits"], wl["token"], wl["parent"], wl["node_off"], cap,
+                        bf16=wl["logits"].dtype == np.uint16)
+        for g, r in zip(got, want):
+            np.testing.assert_array_equal(g.cpu().numpy(), r)
+
+
+def test_accept_noalloc_rows_outside_every_tree():
+    """A node_off whose last entry falls short of n_total leaves rows in no
+    tree: they raise TG_ERR_DEVICE_TREE instead of drawing a ticket of the
+    last tree, and the next call is exact again."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_26112_gb300 import build
+    build.build()
+    import paper_2608_26112_gb300 as tg
+    lib = tg.lib()
+    dev = torch.device("cuda:0")
+    logits, token, parent, node_off, B, max_nodes, n_total = _inputs("llama3-70b-verify", 9, dev)
+    short = node_off.clone()
+    short[-1] -= 3
+    _noalloc_call(lib, logits, token, parent, short, B, max_nodes, n_total, max_nodes)
+    assert tg.last_device_status() & 4
+    got = _noalloc_call(lib, logits, token, parent, node_off, B, max_nodes, n_total, max_nodes)
+    ws = tg.accept_workspace(B, n_total, dev)
+    ref = tg.accept(logits, token, parent, node_off, max_nodes, max_nodes, ws)
+    assert tg.last_device_status() == 0
+    for g, r in zip(got, ref):
+        assert torch.equal(g, r)
 
 
 def test_accept_noalloc_rejects_sizes_beyond_its_array():
