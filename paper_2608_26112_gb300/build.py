@@ -16,7 +16,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libtreegraft.so")
-SOURCES = ["api.cu", "tree_attn.cu", "topk.cu", "accept.cu", "rescore.cu", "accept_noalloc.cu",
+SOURCES = ["api.cu", "tree_attn.cu", "tree_attn_split.cu", "topk.cu", "accept.cu", "rescore.cu", "accept_noalloc.cu",
            "prune.cu", "grow.cu", "ngram.cu", "sample.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",

@@ -128,7 +128,8 @@ extern "C" {
 
 size_t treegraft_tree_attn_workspace_size(int B, int max_nodes, int Hq, int Hkv, int D) {
   if (B < 1 || max_nodes < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || (D != 64 && D != 128)) return 0;
-  return tree_attn_ws_bytes(D, B, Hkv, Hq / Hkv, max_nodes);
+  const int mtiles = ((Hq / Hkv) * max_nodes + 127) / 128;
+  return tree_attn_split_ws_bytes(D, B, Hkv, mtiles, kAttnMaxSplits);
 }
 
 int treegraft_set_wait_budget(int64_t cycles) {
@@ -159,12 +160,13 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
   int* st = status_ptr();
   if (!st) return TG_ERR_CUDA;
 
-  CUtensorMap tq, tk, tv;
+  CUtensorMap tq, tk, tv, to;
   {
     const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hq, (cuuint64_t)n_total};
     const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hq * D * 2};
     const cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(128 / G)};
     if (!encode_bf16(&tq, q, 3, dims, strides, box)) return TG_ERR_CUDA;
+    if (!encode_bf16(&to, out, 3, dims, strides, box)) return TG_ERR_CUDA;  // same box as q
   }
   {
     const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)B * Hkv * S_max};
@@ -189,20 +191,39 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
   a.out = out;
   a.lse_out = lse_out;
   a.status = st;
-  const AttnPlan plan = tree_attn_plan(D, B, Hkv, G, max_nodes, S_max, device_sm_count());
-  a.unit_rows = plan.unit_rows;
-  a.rblocks = tree_attn_rblocks(G, max_nodes, plan.unit_rows);
-  if (plan.splits > 1) {
-    const size_t need = tree_attn_ws_bytes(D, B, Hkv, G, max_nodes);
-    if (ws == nullptr || ws_bytes < need || !aligned16(ws)) return TG_ERR_INVALID_ARG;
-  }
-  a.ws = ws;
-  a.lpt = plan.lpt;
   a.split_wait_cycles = g_wait_budget.load();
-  return launch_tree_attn(tq, tk, tv, a, plan, static_cast<cudaStream_t>(stream)) == cudaSuccess
-             ? TG_OK
-             : TG_ERR_CUDA;
+  // Two kernels, one per regime: the split kernel for small problems (keys
+  // of a 128-row work item split over several CTAs, partials combined
+  // through the workspace), the two-tile kernel for whole units once there
+  // are enough of them to fill the GPU.  Each plan estimates its launch
+  // time; the cheaper one runs.
+  const int nsm = device_sm_count();
+  const int mtiles = (G * max_nodes + 127) / 128;
+  double split_cost = 0.0;
+  const SplitPlan sp = tree_attn_split_plan(D, B, Hkv, mtiles, S_max, nsm, &split_cost);
+  const WholePlan wp = tree_attn_whole_plan(D, B, Hkv, G, max_nodes, S_max, nsm);
+  const cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  // With a wave of work items or more there is nothing to split: whole
+  // units in longest-first order (ragged batches) are then the better plan.
+  const bool full = (long long)B * Hkv * mtiles >= nsm;
+  if (wp.cost_us < split_cost || (B > 1 && full)) {
+    a.unit_rows = wp.unit_rows;
+    a.rblocks = tree_attn_rblocks(G, max_nodes, wp.unit_rows);
+    a.lpt = wp.lpt;
+    a.ws = nullptr;
+    a.coop = 0;
+    return launch_tree_attn(tq, tk, tv, to, a, cs) == cudaSuccess ? TG_OK : TG_ERR_CUDA;
+  }
+  const size_t need = tree_attn_split_ws_bytes(D, B, Hkv, mtiles, sp.splits);
+  if (need > 0 && (ws == nullptr || ws_bytes < need || !aligned16(ws))) return TG_ERR_INVALID_ARG;
+  a.ws = ws;
+  a.coop = sp.coop;
+  a.unit_rows = 128;
+  a.rblocks = mtiles;
+  a.lpt = 0;
+  return launch_tree_attn_split(tq, tk, tv, a, sp, cs) == cudaSuccess ? TG_OK : TG_ERR_CUDA;
 }
+
 
 int treegraft_expand_topk(const void* logits, int dtype, int logit_rows, int V, int64_t ld,
                           int rows, const int32_t* row_idx, const float* parent_score, int k,

@@ -13,36 +13,48 @@ struct AttnArgs {
   const int32_t* parent;
   const int32_t* node_off;
   int B, max_nodes, n_total, Hq, Hkv, D, S_max;
-  int unit_rows;     // query rows per work unit: 256 (two tiles) or 128 (one)
-  int rblocks;       // units per (tree, kv-head) at max_nodes
   float scale_log2;  // softmax scale * log2(e)
   void* out;
   float* lse_out;
-  void* ws;  // split counters + combine partial rows (tree_attn_ws_bytes)
   int* status;
-  int lpt;   // 1: one CTA per unit, units dealt longest tree first (1-D grid)
-  long long split_wait_cycles;  // bound of the wait on the other splits of a unit
+  // two-tile kernel (tree_attn.cu): whole units
+  int unit_rows;     // query rows per work unit: 256 (two tiles) or 128 (one)
+  int rblocks;       // units per (tree, kv-head) at max_nodes
+  int lpt;           // 1: units dealt longest tree first (trees ranked on the device)
+  // split kernel (tree_attn_split.cu)
+  void* ws;          // split counters + combine partial rows (tree_attn_split_ws_bytes)
+  int coop;          // 1: cooperative launch, split barrier on counters in ws; 0: clusters
+  long long split_wait_cycles;  // bound of the wait on the other splits of a work item
 };
-// How one launch cuts the work: `splits` CTAs per unit (the key tiles dealt
-// round-robin; > 1 needs a cooperative launch whose whole grid is resident
-// at once), and whether units are dealt longest tree first.
-struct AttnPlan {
-  int splits;
-  int lpt;
+// two-tile kernel: one CTA per unit, every key tile
+struct WholePlan {
   int unit_rows;
+  int lpt;
+  double cost_us;  // estimated launch time
 };
-constexpr int kAttnMaxSplits = 32;
+cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
+                             const CUtensorMap& tm_v, const CUtensorMap& tm_o, const AttnArgs& a,
+                             cudaStream_t s);
+int tree_attn_rblocks(int G, int max_nodes, int unit_rows);
+WholePlan tree_attn_whole_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max,
+                               int num_sms);
+// split kernel: `splits` CTAs per 128-row work item, joined by a thread-block
+// cluster or, with coop, by a cooperative launch whose whole grid is resident
+struct SplitPlan {
+  int splits;
+  int coop;
+};
+cudaError_t launch_tree_attn_split(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
+                                   const CUtensorMap& tm_v, const AttnArgs& a, SplitPlan plan,
+                                   cudaStream_t s);
+SplitPlan tree_attn_split_plan(int D, int B, int Hkv, int mtiles, int S_max, int num_sms,
+                               double* cost_us);
+size_t tree_attn_split_ws_bytes(int D, int B, int Hkv, int mtiles, int splits);
+constexpr int kAttnMaxSplits = 10;
 // default bound of the waits on other thread blocks: about one second at the
 // GB300's maximum SM clock (the same bound as the in-block mbarrier waits)
 constexpr long long kInterBlockWaitCycles = 2000000000LL;
-constexpr int kAttnMaxCoopCtas = 256;  // split plans never exceed this many CTAs
-// tmaps: q [D, Hq, n_total], k and v [D, B*Hkv*S_max] (innermost first)
-cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
-                             const CUtensorMap& tm_v, const AttnArgs& a, AttnPlan plan,
-                             cudaStream_t s);
-int tree_attn_rblocks(int G, int max_nodes, int unit_rows);
-AttnPlan tree_attn_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max, int num_sms);
-size_t tree_attn_ws_bytes(int D, int B, int Hkv, int G, int max_nodes);
+// tmaps: q and out [D, Hq, n_total], k and v [D, B*Hkv*S_max] (innermost first)
 
 struct TopkArgs {
   const void* logits;

@@ -28,17 +28,14 @@
 //               in TMEM only when the row max grows by more than 8 (base 2)
 //               past the reference its P values were taken against.
 //
-// Launch plans (chosen on the host by tree_attn_plan):
-//   split   the key tiles of a unit are dealt round-robin to S CTAs of a
-//           cooperative launch (the whole grid resident at once).  Each CTA
-//           writes its partial rows (O / l in bf16, max and sum in fp32) to
-//           the caller's workspace, the S CTAs of a unit meet on a counter
-//           there, and each merges a slice of the unit's rows;
-//   whole   one CTA per unit with every key tile, output written straight
-//           from TMEM.  For batches of several trees the units are dealt in
-//           longest-tree-first order (a ranking every CTA computes from
-//           prefix_len and node_off), so ragged batches end together.
-// Every mbarrier wait is bounded, and so is the split counter wait.
+// One CTA computes a whole unit (every key tile) and writes its output rows
+// straight from TMEM.  The host sends launches here when there are enough
+// units to fill the GPU (large or batched verification: the Llama-3-70B
+// shape, serving batches); small problems whose keys must be split over
+// several CTAs go to tree_attn_split.cu.  For batches of several trees the
+// units are dealt in longest-tree-first order (a ranking every CTA computes
+// from prefix_len and node_off), so ragged batches end together.
+// Every mbarrier wait is bounded.
 #include <algorithm>
 
 #include "common.cuh"
@@ -84,18 +81,11 @@ struct Layout {
   static constexpr int kOffMisc = align_up(kOffBar + kNumBars * 8, 16);  // tmem addr, flags, unit
   static constexpr int kBytes = kOffMisc + 64;
   static constexpr int kAlloc = kBytes + 1024;  // 1024-byte alignment slack
-  // One CTA's partial rows in the workspace: O / l as bf16 in [D / 8][kRows]
-  // groups of 8 (a warp's 32 rows are 512 contiguous bytes), then m[kRows]
-  // (base 2) and l[kRows] (fp32).
-  static constexpr int kSlabBytes = kRows * (2 * D + 8);
-  static constexpr int kSlabM = kRows * D * 2;
-  static constexpr int kSlabL = kSlabM + kRows * 4;
   static_assert(kAlloc <= 227 * 1024, "shared memory budget");
   static_assert(kOffQ % 1024 == 0 && kOffK % 1024 == 0 && kOffV % 1024 == 0,
                 "128-byte-swizzled operand tiles need 1024-byte alignment");
   static_assert(kOffBar % 8 == 0 && kOffMisc % 16 == 0, "mbarrier / scalar alignment");
   static_assert(kAncRows * kAncWords * 4 >= 3 * kLptMaxTrees * 4, "ranking scratch");
-  static_assert(kSlabBytes % 16 == 0 && kSlabM % 16 == 0, "16-byte slab groups");
 };
 
 // 32 mask bits of one node for tree slots [b0, b0 + 32): slot < 0 is the
@@ -168,20 +158,6 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 // id 0 is __syncthreads)
 __device__ __forceinline__ void group_bar(int g) {
   asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "n"(kGroup) : "memory");
-}
-
-// Workspace: two int counters per unit (the split barrier), padded to 256
-// bytes, then the partial-row slabs.
-__host__ __device__ constexpr size_t attn_counter_bytes(long long units) {
-  return (size_t)((units * 8 + 255) / 256 * 256);
-}
-__device__ __forceinline__ void red_add_release_gpu(int* p, int v) {
-  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
 }
 
 // Which unit this CTA computes in a longest-first launch: trees ranked by
@@ -257,93 +233,20 @@ __device__ void lpt_unit(const AttnArgs& a, int G, long long slot, int* scratch,
   __syncthreads();
 }
 
-// Merge the S partial rows of the rows this CTA owns (Sec. 3.1 attention as
-// a softmax over the union of the splits' keys).  Split s holds O_s / l_s
-// (bf16), its max m_s (base 2) and sum l_s: with w_s = 2^(m_s - M) l_s,
-// M = max_s m_s, the row is o = sum_s w_s (O_s / l_s) / sum_s w_s and
-// lse = ln 2 (M + log2 sum_s w_s).  A running (M, sum, acc) takes the splits
-// four at a time, with the four splits' loads in flight together.
-template <int D>
-__device__ void combine_rows(const char* slabs, int S, int split, int rows, int rb, int G,
-                             int n, int off, int h, const AttnArgs& a) {
-  using L = Layout<D>;
-  const float NEG_INF = __int_as_float(0xff800000);
-  const int rpc = (rows + S - 1) / S;
-  const int row_lo = split * rpc;
-  const int my_rows = max(0, min(rows, row_lo + rpc) - row_lo);
-  constexpr int CG = D / 8;
-  for (int item = threadIdx.x; item < my_rows * CG; item += kThreads) {
-    const int ur = row_lo + item % my_rows, c8 = item / my_rows;
-    const int rg = rb * a.unit_rows + ur;
-    const int uu = rg / G, g = rg % G;
-    if (uu >= n) continue;
-    float M = NEG_INF, Ls = 0.f;
-    float acc[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-    constexpr int kBatch = 16;  // splits whose loads are in flight together
-    for (int s0 = 0; s0 < S; s0 += kBatch) {
-      float mv[kBatch], lv[kBatch];
-      uint4 ov[kBatch];
-#pragma unroll
-      for (int j = 0; j < kBatch; ++j) {
-        mv[j] = NEG_INF;
-        lv[j] = 0.f;
-        ov[j] = make_uint4(0u, 0u, 0u, 0u);
-        if (s0 + j < S) {
-          const char* src = slabs + (size_t)(s0 + j) * L::kSlabBytes;
-          mv[j] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabM) + ur);
-          lv[j] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabL) + ur);
-          ov[j] = __ldcg(reinterpret_cast<const uint4*>(src) + (size_t)c8 * kRows + ur);
-        }
-      }
-      float Mb = M;
-#pragma unroll
-      for (int j = 0; j < kBatch; ++j) Mb = fmaxf(Mb, mv[j]);
-      if (Mb == NEG_INF) continue;
-      if (Mb > M) {
-        const float c = (M == NEG_INF) ? 0.f : ex2(M - Mb);
-        Ls *= c;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) acc[q] *= c;
-        M = Mb;
-      }
-#pragma unroll
-      for (int j = 0; j < kBatch; ++j) {
-        const float w = (mv[j] == NEG_INF) ? 0.f : ex2(mv[j] - M) * lv[j];
-        Ls += w;
-        const uint32_t wd[4] = {ov[j].x, ov[j].y, ov[j].z, ov[j].w};
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          acc[2 * q] = fmaf(w, __uint_as_float(wd[q] << 16), acc[2 * q]);
-          acc[2 * q + 1] = fmaf(w, __uint_as_float(wd[q] & 0xFFFF0000u), acc[2 * q + 1]);
-        }
-      }
-    }
-    const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
-    const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
-    uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c8 * 8);
-    *dst = make_uint4(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv),
-                      pack_bf16(acc[4] * inv, acc[5] * inv), pack_bf16(acc[6] * inv, acc[7] * inv));
-    if (c8 == 0 && a.lse_out) a.lse_out[orow] = (M == NEG_INF) ? M : (M + log2f(Ls)) * kLn2;
-  }
-}
-
 template <int D>
 __global__ void __maxnreg__(168)
     tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                      const __grid_constant__ CUtensorMap tm_k,
-                     const __grid_constant__ CUtensorMap tm_v, const AttnArgs a) {
+                     const __grid_constant__ CUtensorMap tm_v,
+                     const __grid_constant__ CUtensorMap tm_o, const AttnArgs a) {
   using L = Layout<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = a.Hq / a.Hkv;
-  // split plan: x = split, y = unit (b, h, rb with rb fastest); whole plan
-  // with lpt: x = slot in longest-first order
-  const int S_kv = a.lpt ? 1 : (int)gridDim.x;
-  const int split = a.lpt ? 0 : (int)blockIdx.x;
+  // x = unit: (b, h, rb) with rb fastest, or with lpt the slot in
+  // longest-first order.  The key tiles of a unit all belong to this CTA.
 
   int* par_s = reinterpret_cast<int*>(smem + L::kOffPar);
   uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + L::kOffAnc);
@@ -363,19 +266,19 @@ __global__ void __maxnreg__(168)
 
   int b = 0, h = 0, rb = 0;
   if (!a.lpt) {
-    const int ui = blockIdx.y;
+    const int ui = blockIdx.x;
     b = ui / (a.Hkv * a.rblocks);
     h = (ui / a.rblocks) % a.Hkv;
     rb = ui % a.rblocks;
   }
-  // ---- barriers; in a split plan the first K/V copies (and tree 0's Q
+  // ---- barriers; in unit order the first K/V copies (and tree 0's Q
   //      tiles, which start at node 0) go out before any global read returns
   const int kv_rows = a.B * a.Hkv * a.S_max;
   auto kv_row0 = [&]() { return (b * a.Hkv + h) * a.S_max; };
-  auto load_k = [&](int it) {  // it-th tile of this split = tile split + it * S_kv
+  auto load_k = [&](int it) {  // it-th key tile of the unit
     const int st = it & 1;
     mbar_arrive_expect_tx(bar(BAR_K_FULL + st), L::kKVBytes);
-    const int y = kv_row0() + (split + it * S_kv) * kBN;
+    const int y = kv_row0() + it * kBN;
 #pragma unroll
     for (int c = 0; c < D / 64; ++c)
       tma_load_2d(k_base + st * L::kKVBytes + c * kRegion, &tm_k, c * 64, y, bar(BAR_K_FULL + st));
@@ -383,7 +286,7 @@ __global__ void __maxnreg__(168)
   auto load_v = [&](int it) {
     const int st = it & 1;
     mbar_arrive_expect_tx(bar(BAR_V_FULL + st), L::kKVBytes);
-    const int y = kv_row0() + (split + it * S_kv) * kBN;
+    const int y = kv_row0() + it * kBN;
 #pragma unroll
     for (int c = 0; c < D / 64; ++c)
       tma_load_2d(v_base + st * L::kKVBytes + c * kRegion, &tm_v, c * 64, y, bar(BAR_V_FULL + st));
@@ -410,7 +313,7 @@ __global__ void __maxnreg__(168)
   int q_early = 0;  // tile mask
 #pragma unroll
   for (int s = 0; s < kStages; ++s)
-    kv_early[s] = !a.lpt && kv_row0() + (split + s * S_kv) * kBN < kv_rows;
+    kv_early[s] = !a.lpt && kv_row0() + s * kBN < kv_rows;
   if (!a.lpt && b == 0)
     for (int t = 0; t < kQT; ++t)
       if (t * kBM < a.unit_rows && (rb * a.unit_rows + t * kBM) / G < a.n_total) q_early |= 1 << t;
@@ -435,7 +338,7 @@ __global__ void __maxnreg__(168)
     if (q_early) load_q(0, q_early);
 #pragma unroll
     for (int s = 0; s < kStages; ++s)
-      if (kv_early[s]) {  // used when this split has that many tiles
+      if (kv_early[s]) {  // used when the unit has that many tiles
         load_k(s);
         load_v(s);
       }
@@ -474,7 +377,7 @@ __global__ void __maxnreg__(168)
   const bool two = rows > kBM;  // query tile 1 holds rows
   const int Lk = P + n;
   const int T = (Lk + kBN - 1) / kBN;
-  const int nt = skip ? 0 : (split < T ? (T - split + S_kv - 1) / S_kv : 0);
+  const int nt = skip ? 0 : T;  // key tiles of the unit
   if (tid == 0 && !q_early && nt > 0) load_q(off, two ? 3 : 1);
   tc_fence_before();
   __syncthreads();
@@ -491,10 +394,8 @@ __global__ void __maxnreg__(168)
         }
       if (q_early) ok = mbar_wait(bar(BAR_Q_FULL), 0) && ok;
       if (!ok) raise_status(a.status, kStTimeout);
-      if (bad_shape && split == 0 && rb == 0) raise_status(a.status, kStTree);
+      if (bad_shape && rb == 0 && h == 0) raise_status(a.status, kStTree);
     }
-    // (uniform over the unit: every split of it skips, and none of them
-    // touches the unit's counter)
     __syncthreads();
     if (warp == 1) tmem_dealloc(tmem, 512);
     return;
@@ -622,14 +523,14 @@ __global__ void __maxnreg__(168)
     // both groups meet once: parent array and validity are shared
     asm volatile("bar.sync 3, %0;" ::"n"(kQT * kGroup) : "memory");
     const bool tree_ok = misc[5] == 0;
-    if (!tree_ok && gt == 0 && split == 0 && rb == 0) raise_status(a.status, kStTree);
+    if (!tree_ok && gt == 0 && rb == 0 && h == 0) raise_status(a.status, kStTree);
     const uint32_t* anc = anc_s + (u < n ? (u - u_lo) : (kAncRows - 1)) * kAncWords;
-    // The split's last tile is its only one that can hold tree keys.  If it
-    // does, each group builds its nodes' ancestor bitmasks now, before any
-    // bounded wait, so every warp of the group meets the group barriers
-    // (walk parent pointers to the root, Algorithm 3; a malformed tree keeps
-    // every tree slot masked, its outputs undefined).
-    if (nt > 0 && row_live && (split + (nt - 1) * S_kv) * kBN + kBN > P) {
+    // The unit's last key tile holds the tree's own keys: each group builds
+    // its nodes' ancestor bitmasks now, before any bounded wait, so every
+    // warp of the group meets the group barriers (walk parent pointers to
+    // the root, Algorithm 3; a malformed tree keeps every tree slot masked,
+    // its outputs undefined).
+    if (nt > 0 && row_live) {
       const int n_lo = (g * kBM) / G, n_hi = min((g + 1) * kBM / G, n - u_lo);
       for (int i = n_lo * kAncWords + r; i < n_hi * kAncWords; i += kGroup) anc_s[i] = 0u;
       if (g == 0 && r < kAncWords) anc_s[(kAncRows - 1) * kAncWords + r] = 0u;
@@ -646,7 +547,7 @@ __global__ void __maxnreg__(168)
     bool ok = true;
     for (int it = 0; it < nt && row_live; ++it) {
       const int st = it & 1, ph = it & 1;
-      const int key0 = (split + it * S_kv) * kBN;  // first key of the tile
+      const int key0 = it * kBN;  // first key of the tile
       ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_S_FULL + g), ph));
       if (!ok) break;
       tc_fence_after();
@@ -770,59 +671,69 @@ __global__ void __maxnreg__(168)
     const bool live = have && m_out != NEG_INF;
     const uint32_t to = tmem + 256u + (uint32_t)(tile * D) + lane_off;
     const float inv = (live && l_out > 0.f) ? 1.f / l_out : 0.f;
-    if (S_kv == 1) {
-      // ---- whole unit: normalise this row's O and write it
+      // ---- whole unit: normalise this row's O and write it.  A tile whose
+      // 128 rows all lie in the tree (and head size 128, so each group owns
+      // whole 64-column regions) is staged in the consumed stage-0 K / V
+      // buffers in the TMA box layout (128-byte swizzle) and written by
+      // bulk tensor stores, one per region: coalesced, asynchronous.  Other
+      // tiles are stored row by row.
       const size_t orow = (size_t)(off + uw) * a.Hq + (size_t)(h * G + gq);
-      for (int c = c_lo; c < c_hi; ++c) {
-        float o[32];
-        if (have) {
-          tmem_ld32f(to + c * 32, o);
-          tc_wait_ld();
+      float o[D];  // this thread's O columns [32 c_lo, 32 c_hi), loaded together
+      const int nch = c_hi - c_lo;
+#pragma unroll
+      for (int cc = 0; cc < D / 32; ++cc)
+        if (have && cc < nch)
+          tmem_ld32f(to + (c_lo + cc) * 32, *reinterpret_cast<float(*)[32]>(&o[32 * cc]));
+      if (have) tc_wait_ld();
+      const int tile_row0 = rb * a.unit_rows + tile * kBM;  // first query row of the tile
+      const bool full_tile = D == 128 && tile_row0 + kBM <= G * n && (tile == 0 || two);
+      if (full_tile) {
+        // group g stages into its own buffer: tile 1's group (or, with one
+        // tile, the group of region 1) uses V stage 0, the other K stage 0
+        const uint32_t stage = (two ? (g == 0 ? k_base : v_base) : k_base);
+#pragma unroll
+        for (int cc = 0; cc < D / 32; ++cc) {
+          if (cc >= nch) break;
+          const int c = c_lo + cc;                  // 32-column chunk
+          const uint32_t region = stage + (uint32_t)((c >> 1) * kRegion) + (uint32_t)r * 128u;
+          const float* oc = &o[32 * cc];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int j = (c & 1) * 4 + q;          // 16-byte chunk within the 128-byte row
+            const uint4 v4 = make_uint4(pack_bf16(oc[8 * q + 0] * inv, oc[8 * q + 1] * inv),
+                                        pack_bf16(oc[8 * q + 2] * inv, oc[8 * q + 3] * inv),
+                                        pack_bf16(oc[8 * q + 4] * inv, oc[8 * q + 5] * inv),
+                                        pack_bf16(oc[8 * q + 6] * inv, oc[8 * q + 7] * inv));
+            st_shared_v4(region + (uint32_t)(((j ^ (r & 7)) << 4)), live ? v4 : make_uint4(0u, 0u, 0u, 0u));
+          }
         }
-        if (store) {
+        fence_proxy_async_smem();  // generic stores -> bulk copy engine
+        group_bar(g);
+        if (r == 0) {
+          const int node0 = off + tile_row0 / G;
+          for (int c2 = c_lo / 2; c2 < (c_hi + 1) / 2; ++c2)
+            tma_store_3d(&tm_o, stage + (uint32_t)(c2 * kRegion), c2 * 64, h * G, node0);
+          bulk_commit();
+          bulk_wait_read0();  // the staging buffer is read before the CTA moves on
+        }
+      } else if (store) {
+#pragma unroll
+        for (int cc = 0; cc < D / 32; ++cc) {
+          if (cc >= nch) break;
+          const int c = c_lo + cc;
+          const float* oc = &o[32 * cc];
           uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c * 32);
 #pragma unroll
           for (int q = 0; q < 4; ++q)
-            dst[q] = live ? make_uint4(pack_bf16(o[8 * q + 0] * inv, o[8 * q + 1] * inv),
-                                       pack_bf16(o[8 * q + 2] * inv, o[8 * q + 3] * inv),
-                                       pack_bf16(o[8 * q + 4] * inv, o[8 * q + 5] * inv),
-                                       pack_bf16(o[8 * q + 6] * inv, o[8 * q + 7] * inv))
+            dst[q] = live ? make_uint4(pack_bf16(oc[8 * q + 0] * inv, oc[8 * q + 1] * inv),
+                                       pack_bf16(oc[8 * q + 2] * inv, oc[8 * q + 3] * inv),
+                                       pack_bf16(oc[8 * q + 4] * inv, oc[8 * q + 5] * inv),
+                                       pack_bf16(oc[8 * q + 6] * inv, oc[8 * q + 7] * inv))
                           : make_uint4(0u, 0u, 0u, 0u);
         }
       }
       if (store && c_lo == 0 && a.lse_out)
         a.lse_out[orow] = live ? (m_out * sl2 + log2f(l_out)) * kLn2 : NEG_INF;
-    } else {
-      // ---- this row's partial into the workspace, read back after the
-      //      split barrier: O / l as bf16 plus (m base 2, l) in fp32
-      const size_t unit = blockIdx.y;
-      char* slab = reinterpret_cast<char*>(a.ws) + attn_counter_bytes(gridDim.y) +
-                   (unit * (size_t)S_kv + (size_t)split) * L::kSlabBytes;
-      uint4* slab8 = reinterpret_cast<uint4*>(slab);  // [D / 8][kRows] groups of 8 bf16
-      // tcgen05.ld / wait::ld are warp-collective: the condition must be the
-      // same for the 32 lanes (have is)
-      for (int c = c_lo; c < c_hi; ++c) {
-        float o[32];
-        if (have) {
-          tmem_ld32f(to + c * 32, o);
-          tc_wait_ld();
-        }
-        if (store) {
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            __stcg(slab8 + (c * 4 + q) * kRows + urw,
-                   live ? make_uint4(pack_bf16(o[8 * q + 0] * inv, o[8 * q + 1] * inv),
-                                     pack_bf16(o[8 * q + 2] * inv, o[8 * q + 3] * inv),
-                                     pack_bf16(o[8 * q + 4] * inv, o[8 * q + 5] * inv),
-                                     pack_bf16(o[8 * q + 6] * inv, o[8 * q + 7] * inv))
-                        : make_uint4(0u, 0u, 0u, 0u));
-        }
-      }
-      if (store && c_lo == 0) {
-        __stcg(reinterpret_cast<float*>(slab + L::kSlabM) + urw, live ? m_out * sl2 : NEG_INF);
-        __stcg(reinterpret_cast<float*>(slab + L::kSlabL) + urw, live ? l_out : 0.f);
-      }
-    }
   }
   if (tid == 0) {
     // speculative K/V and Q copies this CTA did not consume land in buffers
@@ -840,68 +751,29 @@ __global__ void __maxnreg__(168)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
-  if (S_kv == 1) return;
-
-  // ---- combine through L2.  The S_kv CTAs of a unit meet on a counter in
-  // the workspace: thread 0 adds with release semantics (after the block
-  // barrier, so it covers every thread's stores) and waits, bounded, until
-  // all S_kv have arrived (acquire).
-  const size_t unit = blockIdx.y;
-  if (tid == 0) {
-    int* cnt = reinterpret_cast<int*>(a.ws) + 2 * unit;
-    red_add_release_gpu(cnt, 1);
-    const long long t0 = clock64();
-    bool ok = true;
-    while (ld_acquire_gpu(cnt) < S_kv) {
-      if (clock64() - t0 > a.split_wait_cycles) {
-        ok = false;
-        break;
-      }
-      __nanosleep(32);  // the other splits' release adds reach the line between polls
-    }
-    if (!ok) raise_status(a.status, kStTimeout);
-    // every CTA of the unit has passed the wait once the second counter
-    // reaches S_kv: its last arrival returns both counters to zero for the
-    // next launch
-    if (atomicAdd(cnt + 1, 1) == S_kv - 1) {
-      atomicExch(cnt, 0);
-      atomicExch(cnt + 1, 0);
-    }
-  }
-  __syncthreads();
-  const char* slabs = reinterpret_cast<const char*>(a.ws) + attn_counter_bytes(gridDim.y) +
-                      unit * (size_t)S_kv * L::kSlabBytes;
-  combine_rows<D>(slabs, S_kv, split, rows, rb, G, n, off, h, a);
 }
 
 template <int D>
 cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                     const AttnArgs& a, AttnPlan plan, cudaStream_t s) {
+                     const CUtensorMap& to, const AttnArgs& a, cudaStream_t s) {
   using L = Layout<D>;
   auto kern = tree_attn_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc);
   if (e != cudaSuccess) return e;
   const long long units = (long long)a.B * a.Hkv * a.rblocks;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = a.lpt ? dim3((unsigned)units, 1, 1) : dim3(plan.splits, (unsigned)units, 1);
+  cfg.gridDim = dim3((unsigned)units, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = L::kAlloc;
   cfg.stream = s;
   // programmatic dependent launch: this launch is dispatched while the
   // previous kernel on the stream finishes (its reads wait in the kernel)
-  cudaLaunchAttribute attr[2];
-  int na = 0;
-  if (plan.splits > 1) {
-    attr[na].id = cudaLaunchAttributeCooperative;
-    attr[na].val.cooperative = 1;
-    ++na;
-  }
-  attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[na].val.programmaticStreamSerializationAllowed = 1;
-  ++na;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = na;
-  return cudaLaunchKernelEx(&cfg, kern, tq, tk, tv, a);
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, tq, tk, tv, to, a);
 }
 
 // CTAs of this kernel resident on one SM
@@ -926,66 +798,38 @@ int tree_attn_rblocks(int G, int max_nodes, int unit_rows) {
   return (G * max_nodes + unit_rows - 1) / unit_rows;
 }
 
-// How to cut the work.  Cost model (microseconds, fitted to measured
-// launches): a CTA costs a fixed part (launch, first loads, epilogue) plus
-// one part per 128-key tile, larger when both query tiles hold rows; a
-// split plan adds the partial-row round trip and the counter barrier, and
-// needs the whole grid resident at once (cooperative launch); a whole-unit
-// plan runs in waves of resident CTAs.  Units of 256 rows (two query tiles
-// sharing each K/V tile) or of 128 rows (one tile; twice the units, half the
-// partial rows per split) are both weighed.  Occupancy is cached per device
-// and head size.
-AttnPlan tree_attn_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max, int num_sms) {
+// Whole-unit plan for this kernel: units of 256 rows (two query tiles
+// sharing each K/V tile) or of 128 rows, and the estimated launch time
+// (microseconds, fitted to measured launches): waves of resident CTAs, each
+// a fixed part plus one part per 128-key tile of its unit (larger when both
+// query tiles hold rows).  Occupancy is cached per device and head size.
+WholePlan tree_attn_whole_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max,
+                               int num_sms) {
   static int bps_cache[64][2] = {};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
   const int di = D == 64 ? 0 : 1;
   int& bps = bps_cache[dev][di];
   if (bps == 0) bps = di ? blocks_per_sm_d<128>() : blocks_per_sm_d<64>();
-  const long long resident =
-      std::min<long long>((long long)(bps > 0 ? bps : 1) * num_sms, kAttnMaxCoopCtas);
+  const long long resident = (long long)(bps > 0 ? bps : 1) * num_sms;
   const int tiles = (S_max + kBN - 1) / kBN;
-  const double kFixed = 3.5, kCombineBase = 1.5, kCombinePerRow = 4.0 / kRows;
-  AttnPlan best{1, 0, kRows};
-  double best_cost = 1e30;
+  const double kFixed = 5.0;
+  WholePlan best{kRows, B > 1 ? 1 : 0, 1e30};
   for (int ur = kRows; ur >= kBM; ur -= kBM) {
-    const int rbm = tree_attn_rblocks(G, max_nodes, ur);
-    const long long units = (long long)B * Hkv * rbm;
+    const long long units = (long long)B * Hkv * tree_attn_rblocks(G, max_nodes, ur);
     const int rows = std::min(ur, G * max_nodes);
-    const double per_tile = rows > kBM ? 1.2 : 0.75;
-    const double whole = (double)((units + resident - 1) / resident) * (kFixed + per_tile * tiles);
-    if (whole < best_cost - 1e-9) {
-      best_cost = whole;
-      best = AttnPlan{1, B > 1 || units > 65535 ? 1 : 0, ur};
-    }
-    if (units > 65535) continue;
-    for (int s = 2; s <= kAttnMaxSplits && s <= tiles; ++s) {
-      if (units * s > resident) break;
-      const double cost = kFixed + kCombineBase + kCombinePerRow * rows +
-                          per_tile * (double)((tiles + s - 1) / s);
-      if (cost < best_cost - 1e-9) {
-        best_cost = cost;
-        best = AttnPlan{s, 0, ur};
-      }
-    }
+    const double per_tile = rows > kBM ? 1.8 : 1.0;
+    const double cost = (double)((units + resident - 1) / resident) * (kFixed + per_tile * tiles);
+    if (cost < best.cost_us - 1e-9) best = WholePlan{ur, B > 1 ? 1 : 0, cost};
   }
   return best;
 }
 
-size_t tree_attn_ws_bytes(int D, int B, int Hkv, int G, int max_nodes) {
-  const size_t slab = D == 64 ? (size_t)Layout<64>::kSlabBytes : (size_t)Layout<128>::kSlabBytes;
-  // the larger unit count (128-row units) bounds both unit sizes
-  const long long units = (long long)B * Hkv * tree_attn_rblocks(G, max_nodes, kBM);
-  const long long slabs = std::min<long long>(units * kAttnMaxSplits, kAttnMaxCoopCtas);
-  if (units > kAttnMaxCoopCtas / 2) return 0;  // never split: at most one CTA per unit resident
-  return attn_counter_bytes(units) + (size_t)slabs * slab;
-}
-
 cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
-                             const CUtensorMap& tm_v, const AttnArgs& a, AttnPlan plan,
+                             const CUtensorMap& tm_v, const CUtensorMap& tm_o, const AttnArgs& a,
                              cudaStream_t s) {
-  if (a.D == 64) return launch_d<64>(tm_q, tm_k, tm_v, a, plan, s);
-  return launch_d<128>(tm_q, tm_k, tm_v, a, plan, s);
+  if (a.D == 64) return launch_d<64>(tm_q, tm_k, tm_v, tm_o, a, s);
+  return launch_d<128>(tm_q, tm_k, tm_v, tm_o, a, s);
 }
 
 }  // namespace tg

@@ -43,16 +43,10 @@ def test_status_strings(lib):
 
 
 def test_tree_attn_workspace_size(lib):
-    # two int counters per (tree, kv-head, 256-row block) padded to 256 bytes, then
-    # one slab of 256 rows x (D bf16 + 2 fp32) per (unit, split): at most 32 splits
-    # and at most 256 slabs (a split launch has all its CTAs resident at once)
-    units = 1 * 8 * 1
-    assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 128) == 256 + units * 32 * 256 * 264
-    units = 2 * 8 * 1
-    assert lib.treegraft_tree_attn_workspace_size(2, 60, 32, 8, 128) == 256 + 256 * 256 * 264
-    assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 64) == 256 + 8 * 32 * 256 * 136
-    # more than 128 units never split: no workspace
-    assert lib.treegraft_tree_attn_workspace_size(5, 128, 64, 8, 128) == 0
+    # two int counters per (tree, kv-head, 128-row work item) padded to 256 bytes, then
+    # per (work item, split) a slab of 128 rows x (D bf16 + 2 fp32), up to 10 splits
+    units = 1 * 8 * 2
+    assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 128) == 256 + units * 10 * 128 * 264
     assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 96) == 0
 
 
