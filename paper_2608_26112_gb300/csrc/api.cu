@@ -129,7 +129,8 @@ extern "C" {
 size_t treegraft_tree_attn_workspace_size(int B, int max_nodes, int Hq, int Hkv, int D) {
   if (B < 1 || max_nodes < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || (D != 64 && D != 128)) return 0;
   const int mtiles = ((Hq / Hkv) * max_nodes + 127) / 128;
-  return tree_attn_split_ws_bytes(D, B, Hkv, mtiles, kAttnMaxSplits);
+  return std::max(tree_attn_split_ws_bytes(D, B, Hkv, mtiles, kAttnMaxSplits),
+                  tree_attn_whole_ws_bytes(D, B, Hkv, Hq / Hkv, max_nodes));
 }
 
 int treegraft_set_wait_budget(int64_t cycles) {
@@ -210,7 +211,13 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
     a.unit_rows = wp.unit_rows;
     a.rblocks = tree_attn_rblocks(G, max_nodes, wp.unit_rows);
     a.lpt = wp.lpt;
-    a.ws = nullptr;
+    // long units are cut into key chunks merged through the workspace when
+    // it is large enough; otherwise every unit stays whole
+    const bool chunks = ws && aligned16(ws) && ws_bytes >= tree_attn_whole_ws_bytes(D, B, Hkv, G, max_nodes);
+    a.ws = chunks ? ws : nullptr;
+    a.slab_off = tree_attn_whole_slab_off(B, Hkv, G, max_nodes);
+    a.resident = tree_attn_whole_resident(D, nsm);
+    a.chunk_min = kWholeChunkMin;
     a.coop = 0;
     return launch_tree_attn(tq, tk, tv, to, a, cs) == cudaSuccess ? TG_OK : TG_ERR_CUDA;
   }

@@ -17,10 +17,13 @@ struct AttnArgs {
   void* out;
   float* lse_out;
   int* status;
-  // two-tile kernel (tree_attn.cu): whole units
+  // two-tile kernel (tree_attn.cu): whole units, long ones cut into key chunks
   int unit_rows;     // query rows per work unit: 256 (two tiles) or 128 (one)
   int rblocks;       // units per (tree, kv-head) at max_nodes
-  int lpt;           // 1: units dealt longest tree first (trees ranked on the device)
+  int lpt;           // 1: items dealt longest first (work list built on the device)
+  int resident;      // CTAs resident at once (the chunk length aims at one item each)
+  int chunk_min;     // shortest key chunk, in 128-key tiles
+  size_t slab_off;   // byte offset of the chunk slabs in ws (after the unit tickets)
   // split kernel (tree_attn_split.cu)
   void* ws;          // split counters + combine partial rows (tree_attn_split_ws_bytes)
   int coop;          // 1: cooperative launch, split barrier on counters in ws; 0: clusters
@@ -38,6 +41,13 @@ cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
 int tree_attn_rblocks(int G, int max_nodes, int unit_rows);
 WholePlan tree_attn_whole_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max,
                                int num_sms);
+// workspace of the two-tile kernel: unit tickets, then the partial-row slabs
+// of the key chunks (at most kWholeMaxSlabs, twice the resident CTAs)
+size_t tree_attn_whole_ws_bytes(int D, int B, int Hkv, int G, int max_nodes);
+size_t tree_attn_whole_slab_off(int B, int Hkv, int G, int max_nodes);
+int tree_attn_whole_resident(int D, int num_sms);
+constexpr int kWholeMaxResident = 256;
+constexpr int kWholeChunkMin = 8;
 // split kernel: `splits` CTAs per 128-row work item, joined by a thread-block
 // cluster or, with coop, by a cooperative launch whose whole grid is resident
 struct SplitPlan {

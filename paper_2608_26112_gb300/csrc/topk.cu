@@ -3,27 +3,27 @@
 // Algorithms 1 and 2), one HBM pass over the logits.
 //
 // Grid (C, rows) with clusters of C CTAs along x: the C CTAs of a cluster
-// split one row.  After the load the selection needs one block barrier and
-// one cluster barrier:
-//   - every CTA stages its chunk in registers (eight 16-byte loads per
-//     thread, all in flight at once) and takes its thread maxima; each warp
-//     finds its top rl lane maxima (rl = ceil(k / 8)); after a block barrier
-//     every warp takes the k-th largest T_c of the CTA's 8 rl maxima.  At
-//     least k elements of the chunk reach T_c, so the chunk's own top-k do,
-//     and the row's top-k lies among the candidates of its CTAs.  Meanwhile
-//     each thread takes the sum of exp(x - max) over its elements (one
-//     exponential per element) and each warp folds its lanes' (max, sum);
-//   - each warp pushes its (max, sum) pair to the cluster's leader, and the
-//     threads whose max reaches T_c visit the 16-byte vectors whose packed
-//     max reaches it and push those elements' 64-bit keys (value desc, token
-//     asc - exact on ties) into the leader's candidate buffer (DSMEM
-//     atomics);
-//   - after the cluster barrier the leader ranks the candidates (about C k)
-//     by counting larger keys, folds the C * 8 (max, sum) pairs into the
-//     lse, and writes token, logprob = x - lse and score = fp32(parent_score
-//     + logprob).  A tie-heavy row that overflows the candidate buffer is
-//     ranked exactly by the leader alone from global memory (k rounds of a
-//     block-wide key max) - slow, rare.
+// split one row.  The selection uses no block barrier, only three phases of
+// the cluster barrier:
+//   0. every CTA stages its chunk in registers (eight 16-byte loads per
+//      thread, all in flight at once) and takes its thread maxima; each warp
+//      finds its top r lane maxima (r = ceil(k / (8 C)), so the row pushes at
+//      least k values) and stores them into EVERY CTA of the cluster (DSMEM);
+//   1. while the other CTAs finish, each thread takes the sum of exp(x - max)
+//      over its elements (packed bf16x2 max, one exp per element), each warp
+//      folds its lanes' (max, sum) with one exponential per lane and pushes
+//      the pair to the leader.  After the barrier every
+//      warp holds the same 8 C r pushed maxima and takes their k-th largest
+//      T: k distinct elements of the row reach T, so the row's top-k all do.
+//      Only threads whose max reaches T hold elements that do; they visit
+//      the 16-byte vectors whose packed max reaches T and push those
+//      elements' 64-bit keys (value desc, token asc - exact on ties) into the
+//      leader's candidate buffer (DSMEM atomics);
+//   2. the leader ranks the few candidates by counting larger keys, folds
+//      the C * 8 (max, sum) pairs into the lse, and writes token, logprob =
+//      x - lse and score = fp32(parent_score + logprob).  A tie-heavy row that
+//      overflows the candidate buffer is ranked exactly by the leader alone
+//      from global memory (k rounds of a block-wide key max) - slow, rare.
 // No global scratch and no second launch.  The kernels are latency-bound
 // after the load, so the code keeps dependency chains short and the
 // executed code small (rare paths are rolled loops).
@@ -40,7 +40,7 @@ namespace {
 constexpr int kMaxK = 32;  // TG_MAX_TOPK
 constexpr int kMaxCluster = 16;
 constexpr int kMaxPush = 128;   // pushed lane maxima per row: 8 C r <= 128
-// rl = ceil(k / 8) <= 4 lane maxima per warp give 8 rl >= k values per CTA
+// r = ceil(k / (8 C)) <= 4 lane maxima per warp give 8 C r >= k pushed values
 static_assert(kMaxK <= 8 * 4 && 8 * kMaxCluster <= kMaxPush, "push sizes");
 constexpr int kCandMax = 2048;  // the leader's candidate buffer
 
@@ -243,7 +243,7 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
     return;
   }
   if (crank == 0 && tid == 0) sm.ncand = 0;
-  // the leader's counter is initialised before any CTA can push
+  // phase 0: the leader's counter is initialised before any CTA can push
   cluster_arrive_release();
   // the leader's threads fetch the parent's path score now, while the
   // logits are in flight (one broadcast request per warp)
@@ -258,28 +258,29 @@ __global__ void __launch_bounds__(kScanThreads, 4) expand_topk_kernel(TopkArgs a
   uint4 buf[kScanVecs];
   scan_load<T, kAligned>(rowp, c0, c1, buf);
   const float tmax = scan_thread_max<T>(buf);
-  // This CTA's threshold: each warp's top rl lane maxima (8 rl >= k values,
-  // every one an element of this CTA's chunk) and their k-th largest T_c.
-  // At least k elements of the chunk reach T_c, so the chunk's own top-k
-  // do, and the row's top-k lies in the union of the CTAs' candidates.  No
-  // cluster exchange is needed to find it, only this block barrier.
-  const int rl = min(4, (k + 7) / 8);
-  const float top = warp_top_r(tmax, rl);
-  if (lane < rl) sm.push_v[warp * rl + lane] = top;
-  // the exp-sum of the row relative to each thread's max, folded per warp
-  float m = tmax, s = scan_thread_sumexp<T>(buf, tmax);
-  warp_lse_pair(m, s);
-  __syncthreads();
-  const float tv = kth_largest_128(sm.push_v, 8 * rl, k);
-  // the leader's counter is initialised and every CTA of the cluster runs:
-  // (max, sum) pairs and candidates go to the leader, then one barrier
+  // each warp's top rp lane maxima go to every CTA of the cluster
+  const int rp = min(4, (k + 8 * C - 1) / (8 * C));
+  const int npush = 8 * C * rp;
+  const float top = warp_top_r(tmax, rp);
   cluster_wait_acquire();
   TopkSmem* lead = cluster.map_shared_rank(&sm, 0);
+  if (lane < rp) {
+    const int slot = (crank * 8 + warp) * rp + lane;
+    for (int c = 0; c < C; ++c) cluster.map_shared_rank(&sm, c)->push_v[slot] = top;
+  }
+  // phase 1: the pushed maxima become visible; the exp-sum runs while the
+  // other CTAs finish their loads
+  cluster_arrive_release();
+  float m = tmax, s = scan_thread_sumexp<T>(buf, tmax);
+  warp_lse_pair(m, s);
   if (lane == 0) {
     lead->recv_m[crank * 8 + warp] = m;
     lead->recv_s[crank * 8 + warp] = s;
   }
+  cluster_wait_acquire();
+  const float tv = kth_largest_128(sm.push_v, npush, k);
   if (tmax >= tv) push_candidates<T>(buf, c0, c1, tv, lead);
+  // phase 2: every candidate and (max, sum) has reached the leader
   cluster_arrive_release();
   cluster_wait_acquire();
   if (crank != 0) return;

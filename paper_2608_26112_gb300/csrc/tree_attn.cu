@@ -78,14 +78,20 @@ struct Layout {
   static constexpr int kOffAnc = kTileEnd;
   static constexpr int kOffPar = align_up(kOffAnc + kAncRows * kAncWords * 4, 16);
   static constexpr int kOffBar = align_up(kOffPar + 256 * 4, 16);
-  static constexpr int kOffMisc = align_up(kOffBar + kNumBars * 8, 16);  // tmem addr, flags, unit
-  static constexpr int kBytes = kOffMisc + 64;
+  static constexpr int kOffMisc = align_up(kOffBar + kNumBars * 8, 16);  // tmem addr, flags, item
+  static constexpr int kBytes = kOffMisc + 80;
   static constexpr int kAlloc = kBytes + 1024;  // 1024-byte alignment slack
   static_assert(kAlloc <= 227 * 1024, "shared memory budget");
   static_assert(kOffQ % 1024 == 0 && kOffK % 1024 == 0 && kOffV % 1024 == 0,
                 "128-byte-swizzled operand tiles need 1024-byte alignment");
   static_assert(kOffBar % 8 == 0 && kOffMisc % 16 == 0, "mbarrier / scalar alignment");
-  static_assert(kAncRows * kAncWords * 4 >= 3 * kLptMaxTrees * 4, "ranking scratch");
+  static_assert(kAncRows * kAncWords * 4 >= 4 * kLptMaxTrees * 4, "ranking scratch");
+  // One chunk's partial rows in the workspace: O / l as bf16 in [D / 8][kRows]
+  // groups of 8 (a warp's 32 rows are 512 contiguous bytes), then m[kRows]
+  // (base 2) and l[kRows] (fp32).
+  static constexpr int kSlabBytes = kRows * (2 * D + 8);
+  static constexpr int kSlabM = kRows * D * 2;
+  static constexpr int kSlabL = kSlabM + kRows * 4;
 };
 
 // 32 mask bits of one node for tree slots [b0, b0 + 32): slot < 0 is the
@@ -160,16 +166,27 @@ __device__ __forceinline__ void group_bar(int g) {
   asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "n"(kGroup) : "memory");
 }
 
-// Which unit this CTA computes in a longest-first launch: trees ranked by
-// (key tiles desc, tree id asc), units of one tree by (kv-head, row block);
-// the slot-th unit of that order.  All threads take part; the result is
-// (b, h, rb) packed in misc[0..2], or b = -1 past the last unit.  Invalid
-// tree extents count as one unit of length 0 (its CTA raises the status).
-__device__ void lpt_unit(const AttnArgs& a, int G, long long slot, int* scratch, int* misc) {
+// The work item this CTA computes in a longest-first launch.  Every CTA
+// derives the same list from prefix_len and node_off: the total work W (key
+// tiles summed over units), a chunk length L = max(chunk_min, ceil(1.25 W /
+// resident CTAs)), and for each tree nch = ceil(tiles / L) key chunks per
+// unit (a unit whose keys are split this way has its chunks merged by the
+// last one to finish).  Trees are ranked by chunk length (desc, tree id asc),
+// items of a tree by (kv-head, row block, chunk); the slot-th item of that
+// order is this CTA's.  All threads take part; the result goes to misc:
+// [0] b (-1 past the last item), [1] h, [2] rb, [3] chunk, [6] chunks of the
+// unit, [7] partial-row slab of the item (-1 for a whole unit).  Invalid
+// tree extents count as one item of length 0 (its CTA raises the status).
+__device__ void lpt_item(const AttnArgs& a, int G, long long slot, int* scratch, int* misc) {
   const int B = a.B;
   int* tiles = scratch;
   int* units = scratch + B;
   int* order = scratch + 2 * B;
+  int* nch = scratch + 3 * B;
+  long long* wsum = reinterpret_cast<long long*>(misc + 8);
+  if (threadIdx.x == 0) *wsum = 0;
+  __syncthreads();
+  long long w = 0;
   for (int t = threadIdx.x; t < B; t += kThreads) {
     const int off = a.node_off[t];
     const int n = a.node_off[t + 1] - off;
@@ -178,59 +195,156 @@ __device__ void lpt_unit(const AttnArgs& a, int G, long long slot, int* scratch,
                     off + n <= a.n_total;
     tiles[t] = ok ? (P + n + kBN - 1) / kBN : 0;
     units[t] = ok ? a.Hkv * ((G * n + a.unit_rows - 1) / a.unit_rows) : 1;
+    w += (long long)tiles[t] * units[t];
   }
+  if (w) atomicAdd(reinterpret_cast<unsigned long long*>(wsum), (unsigned long long)w);
+  __syncthreads();
+  // chunk length: a quarter above the balanced share W / resident, so that
+  // units near the share stay whole (cutting them only adds merges and a
+  // second wave) while the long ones are cut
+  const long long chunk =
+      a.ws ? max((long long)a.chunk_min, (5 * *wsum + 4ll * a.resident - 1) / (4ll * a.resident))
+           : (1ll << 40);
+  for (int t = threadIdx.x; t < B; t += kThreads)
+    nch[t] = tiles[t] > 0 ? (int)((tiles[t] + chunk - 1) / chunk) : 1;
   __syncthreads();
   for (int t = threadIdx.x; t < B; t += kThreads) {
-    const int mine = tiles[t];
+    const int mine = (tiles[t] + nch[t] - 1) / nch[t];
     int rank = 0;
     for (int j = 0; j < B; ++j) {
-      const int o = tiles[j];
+      const int o = (tiles[j] + nch[j] - 1) / nch[j];
       rank += (o > mine || (o == mine && j < t)) ? 1 : 0;
     }
     order[rank] = t;
   }
   __syncthreads();
   if (threadIdx.x < 32) {
-    // inclusive scan of units in rank order, 32 ranks at a time
+    // inclusive scans of items and of split-unit items in rank order, 32
+    // ranks at a time
     const int lane = threadIdx.x;
-    long long carry = 0;
-    int found_b = -1, found_lu = 0;
+    long long carry = 0, carry_s = 0;
+    int found_b = -1, found_li = 0;
+    long long found_slab = 0;
     for (int r0 = 0; r0 < B && found_b < 0; r0 += 32) {
       const int r = r0 + lane;
       const int tb = r < B ? order[r] : 0;
-      long long x = r < B ? units[tb] : 0;
+      const long long items = r < B ? (long long)units[tb] * nch[tb] : 0;
+      const long long sitems = (r < B && nch[tb] > 1) ? items : 0;
+      long long x = items, xs = sitems;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const long long y = __shfl_up_sync(0xffffffffu, x, o);
-        if (lane >= o) x += y;
+        const long long ys = __shfl_up_sync(0xffffffffu, xs, o);
+        if (lane >= o) {
+          x += y;
+          xs += ys;
+        }
       }
-      const long long hi = carry + x;                 // end of this rank's units
-      const long long lo = hi - (r < B ? units[tb] : 0);
+      const long long hi = carry + x;  // end of this rank's items
+      const long long lo = hi - items;
+      const long long slo = carry_s + xs - sitems;  // first slab of this rank's items
       const bool here = r < B && slot >= lo && slot < hi;
       const unsigned m = __ballot_sync(0xffffffffu, here);
       if (m) {
         const int src = __ffs(m) - 1;
         found_b = __shfl_sync(0xffffffffu, tb, src);
-        found_lu = __shfl_sync(0xffffffffu, (int)(slot - lo), src);
+        found_li = __shfl_sync(0xffffffffu, (int)(slot - lo), src);
+        found_slab = __shfl_sync(0xffffffffu, slo, src);
       }
       carry = __shfl_sync(0xffffffffu, hi, 31);
+      carry_s = __shfl_sync(0xffffffffu, carry_s + xs, 31);
     }
     if (lane == 0) {
-      int h = 0, rb = 0;
+      int h = 0, rb = 0, c = 0, nc = 1, slab = -1;
       if (found_b >= 0) {
         const int off = a.node_off[found_b];
         const int n = a.node_off[found_b + 1] - off;
-        const int rbs = max(1, (G * n + a.unit_rows - 1) / a.unit_rows);
         const bool ok = n >= 1 && n <= 256;
-        h = ok ? found_lu / rbs : 0;
-        rb = ok ? found_lu % rbs : 0;
+        const int rbs = max(1, (G * n + a.unit_rows - 1) / a.unit_rows);
+        nc = nch[found_b];
+        const int lu = found_li / nc;
+        c = found_li % nc;
+        h = ok ? lu / rbs : 0;
+        rb = ok ? lu % rbs : 0;
+        if (nc > 1) slab = (int)(found_slab + found_li);
       }
       misc[0] = found_b;
       misc[1] = h;
       misc[2] = rb;
+      misc[3] = c;
+      misc[6] = nc;
+      misc[7] = slab;
     }
   }
   __syncthreads();
+}
+
+// Merge the partial rows of a unit whose keys were split into nc chunks
+// (Sec. 3.1 attention as a softmax over the union of the chunks' keys).
+// Chunk s holds O_s / l_s (bf16), its max m_s (base 2) and sum l_s: with
+// w_s = 2^(m_s - M) l_s, M = max_s m_s, the row is o = sum_s w_s (O_s / l_s)
+// / sum_s w_s and lse = ln 2 (M + log2 sum_s w_s).  Every thread of the CTA
+// takes (row, 8-column group) items; a batch's loads are all in flight at
+// once.
+template <int D>
+__device__ void merge_chunks(const char* slabs, int nc, int rows, int rb, int G, int n, int off,
+                             int h, const AttnArgs& a) {
+  using L = Layout<D>;
+  const float NEG_INF = __int_as_float(0xff800000);
+  constexpr int CG = D / 8;
+  constexpr int kBatch = 8;
+  for (int item = threadIdx.x; item < rows * CG; item += kThreads) {
+    const int ur = item % rows, c8 = item / rows;  // row-fastest: coalesced slab reads
+    const int rg = rb * a.unit_rows + ur;
+    const int uu = rg / G, g = rg % G;
+    if (uu >= n) continue;
+    float M = NEG_INF, Ls = 0.f;
+    float acc[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+    for (int s0 = 0; s0 < nc; s0 += kBatch) {
+      float mv[kBatch], lv[kBatch];
+      uint4 ov[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const char* src = slabs + (size_t)min(s0 + j, nc - 1) * L::kSlabBytes;
+        mv[j] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabM) + ur);
+        lv[j] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabL) + ur);
+        ov[j] = __ldcg(reinterpret_cast<const uint4*>(src) + (size_t)c8 * kRows + ur);
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j)
+        if (s0 + j >= nc) mv[j] = NEG_INF;
+      float Mb = M;
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) Mb = fmaxf(Mb, mv[j]);
+      if (Mb == NEG_INF) continue;
+      if (Mb > M) {
+        const float cf = (M == NEG_INF) ? 0.f : ex2(M - Mb);
+        Ls *= cf;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] *= cf;
+        M = Mb;
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const float wt = (mv[j] == NEG_INF) ? 0.f : ex2(mv[j] - M) * lv[j];
+        Ls += wt;
+        const uint32_t wd[4] = {ov[j].x, ov[j].y, ov[j].z, ov[j].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          acc[2 * q] = fmaf(wt, __uint_as_float(wd[q] << 16), acc[2 * q]);
+          acc[2 * q + 1] = fmaf(wt, __uint_as_float(wd[q] & 0xFFFF0000u), acc[2 * q + 1]);
+        }
+      }
+    }
+    const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
+    const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
+    uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c8 * 8);
+    *dst = make_uint4(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv),
+                      pack_bf16(acc[4] * inv, acc[5] * inv), pack_bf16(acc[6] * inv, acc[7] * inv));
+    if (c8 == 0 && a.lse_out) a.lse_out[orow] = (M == NEG_INF) ? M : (M + log2f(Ls)) * kLn2;
+  }
 }
 
 template <int D>
@@ -265,6 +379,7 @@ __global__ void __maxnreg__(168)
   pdl_wait();
 
   int b = 0, h = 0, rb = 0;
+  int t0 = 0, t1 = 0;  // key tiles [t0, t1) of this CTA's share of the unit
   if (!a.lpt) {
     const int ui = blockIdx.x;
     b = ui / (a.Hkv * a.rblocks);
@@ -278,7 +393,7 @@ __global__ void __maxnreg__(168)
   auto load_k = [&](int it) {  // it-th key tile of the unit
     const int st = it & 1;
     mbar_arrive_expect_tx(bar(BAR_K_FULL + st), L::kKVBytes);
-    const int y = kv_row0() + it * kBN;
+    const int y = kv_row0() + (t0 + it) * kBN;
 #pragma unroll
     for (int c = 0; c < D / 64; ++c)
       tma_load_2d(k_base + st * L::kKVBytes + c * kRegion, &tm_k, c * 64, y, bar(BAR_K_FULL + st));
@@ -286,7 +401,7 @@ __global__ void __maxnreg__(168)
   auto load_v = [&](int it) {
     const int st = it & 1;
     mbar_arrive_expect_tx(bar(BAR_V_FULL + st), L::kKVBytes);
-    const int y = kv_row0() + it * kBN;
+    const int y = kv_row0() + (t0 + it) * kBN;
 #pragma unroll
     for (int c = 0; c < D / 64; ++c)
       tma_load_2d(v_base + st * L::kKVBytes + c * kRegion, &tm_v, c * 64, y, bar(BAR_V_FULL + st));
@@ -347,14 +462,18 @@ __global__ void __maxnreg__(168)
     tmem_alloc(smem_u32(misc + 4), 512);  // S0 [0,128) S1 [128,256) O0 [256,256+D) O1 after
     tmem_relinquish();
   }
+  int chunk = 0, nch = 1, slab = -1;  // key chunk of the unit, chunks, partial-row slab
   if (a.lpt) {
     long long slot = blockIdx.x;
     if (a.B <= kLptMaxTrees) {
-      lpt_unit(a, G, slot, reinterpret_cast<int*>(anc_s), misc);
+      lpt_item(a, G, slot, reinterpret_cast<int*>(anc_s), misc);
       b = misc[0];
       h = misc[1];
       rb = misc[2];
-    } else {  // tree-major order
+      chunk = misc[3];
+      nch = misc[6];
+      slab = misc[7];
+    } else {  // tree-major order, whole units
       b = (int)(slot / ((long long)a.Hkv * a.rblocks));
       h = (int)((slot / a.rblocks) % a.Hkv);
       rb = (int)(slot % a.rblocks);
@@ -377,7 +496,10 @@ __global__ void __maxnreg__(168)
   const bool two = rows > kBM;  // query tile 1 holds rows
   const int Lk = P + n;
   const int T = (Lk + kBN - 1) / kBN;
-  const int nt = skip ? 0 : T;  // key tiles of the unit
+  // key tiles [t0, t1) of this chunk of the unit (all of them when nch = 1)
+  t0 = (int)((long long)chunk * T / nch);
+  t1 = (int)((long long)(chunk + 1) * T / nch);
+  const int nt = skip ? 0 : t1 - t0;
   if (tid == 0 && !q_early && nt > 0) load_q(off, two ? 3 : 1);
   tc_fence_before();
   __syncthreads();
@@ -525,12 +647,12 @@ __global__ void __maxnreg__(168)
     const bool tree_ok = misc[5] == 0;
     if (!tree_ok && gt == 0 && rb == 0 && h == 0) raise_status(a.status, kStTree);
     const uint32_t* anc = anc_s + (u < n ? (u - u_lo) : (kAncRows - 1)) * kAncWords;
-    // The unit's last key tile holds the tree's own keys: each group builds
-    // its nodes' ancestor bitmasks now, before any bounded wait, so every
-    // warp of the group meets the group barriers (walk parent pointers to
-    // the root, Algorithm 3; a malformed tree keeps every tree slot masked,
-    // its outputs undefined).
-    if (nt > 0 && row_live) {
+    // The tree's own keys sit in the unit's last tiles: if this chunk reaches
+    // them, each group builds its nodes' ancestor bitmasks now, before any
+    // bounded wait, so every warp of the group meets the group barriers
+    // (walk parent pointers to the root, Algorithm 3; a malformed tree keeps
+    // every tree slot masked, its outputs undefined).
+    if (nt > 0 && row_live && t1 * kBN > P) {
       const int n_lo = (g * kBM) / G, n_hi = min((g + 1) * kBM / G, n - u_lo);
       for (int i = n_lo * kAncWords + r; i < n_hi * kAncWords; i += kGroup) anc_s[i] = 0u;
       if (g == 0 && r < kAncWords) anc_s[(kAncRows - 1) * kAncWords + r] = 0u;
@@ -547,7 +669,7 @@ __global__ void __maxnreg__(168)
     bool ok = true;
     for (int it = 0; it < nt && row_live; ++it) {
       const int st = it & 1, ph = it & 1;
-      const int key0 = it * kBN;  // first key of the tile
+      const int key0 = (t0 + it) * kBN;  // first key of the tile
       ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_S_FULL + g), ph));
       if (!ok) break;
       tc_fence_after();
@@ -671,69 +793,94 @@ __global__ void __maxnreg__(168)
     const bool live = have && m_out != NEG_INF;
     const uint32_t to = tmem + 256u + (uint32_t)(tile * D) + lane_off;
     const float inv = (live && l_out > 0.f) ? 1.f / l_out : 0.f;
-      // ---- whole unit: normalise this row's O and write it.  A tile whose
-      // 128 rows all lie in the tree (and head size 128, so each group owns
-      // whole 64-column regions) is staged in the consumed stage-0 K / V
-      // buffers in the TMA box layout (128-byte swizzle) and written by
-      // bulk tensor stores, one per region: coalesced, asynchronous.  Other
-      // tiles are stored row by row.
-      const size_t orow = (size_t)(off + uw) * a.Hq + (size_t)(h * G + gq);
-      float o[D];  // this thread's O columns [32 c_lo, 32 c_hi), loaded together
-      const int nch = c_hi - c_lo;
+    // ---- output.  A whole unit normalises its rows and writes them; a
+    // tile whose 128 rows all lie in the tree (head size 128, so each group
+    // owns whole 64-column regions) is staged in the consumed stage-0 K / V
+    // buffers in the TMA box layout (128-byte swizzle) and written by bulk
+    // tensor stores, one per region: coalesced, asynchronous; other tiles
+    // are stored row by row.  A chunk of a split unit writes its partial rows
+    // (O / l in bf16, m base 2, l) to its workspace slab instead.
+    const size_t orow = (size_t)(off + uw) * a.Hq + (size_t)(h * G + gq);
+    float o[D];  // this thread's O columns [32 c_lo, 32 c_hi), loaded together
+    const int n32 = c_hi - c_lo;
 #pragma unroll
-      for (int cc = 0; cc < D / 32; ++cc)
-        if (have && cc < nch)
-          tmem_ld32f(to + (c_lo + cc) * 32, *reinterpret_cast<float(*)[32]>(&o[32 * cc]));
-      if (have) tc_wait_ld();
-      const int tile_row0 = rb * a.unit_rows + tile * kBM;  // first query row of the tile
-      const bool full_tile = D == 128 && tile_row0 + kBM <= G * n && (tile == 0 || two);
-      if (full_tile) {
-        // group g stages into its own buffer: tile 1's group (or, with one
-        // tile, the group of region 1) uses V stage 0, the other K stage 0
-        const uint32_t stage = (two ? (g == 0 ? k_base : v_base) : k_base);
-#pragma unroll
-        for (int cc = 0; cc < D / 32; ++cc) {
-          if (cc >= nch) break;
-          const int c = c_lo + cc;                  // 32-column chunk
-          const uint32_t region = stage + (uint32_t)((c >> 1) * kRegion) + (uint32_t)r * 128u;
-          const float* oc = &o[32 * cc];
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int j = (c & 1) * 4 + q;          // 16-byte chunk within the 128-byte row
-            const uint4 v4 = make_uint4(pack_bf16(oc[8 * q + 0] * inv, oc[8 * q + 1] * inv),
-                                        pack_bf16(oc[8 * q + 2] * inv, oc[8 * q + 3] * inv),
-                                        pack_bf16(oc[8 * q + 4] * inv, oc[8 * q + 5] * inv),
-                                        pack_bf16(oc[8 * q + 6] * inv, oc[8 * q + 7] * inv));
-            st_shared_v4(region + (uint32_t)(((j ^ (r & 7)) << 4)), live ? v4 : make_uint4(0u, 0u, 0u, 0u));
-          }
-        }
-        fence_proxy_async_smem();  // generic stores -> bulk copy engine
-        group_bar(g);
-        if (r == 0) {
-          const int node0 = off + tile_row0 / G;
-          for (int c2 = c_lo / 2; c2 < (c_hi + 1) / 2; ++c2)
-            tma_store_3d(&tm_o, stage + (uint32_t)(c2 * kRegion), c2 * 64, h * G, node0);
-          bulk_commit();
-          bulk_wait_read0();  // the staging buffer is read before the CTA moves on
-        }
-      } else if (store) {
+    for (int cc = 0; cc < D / 32; ++cc)
+      if (have && cc < n32)
+        tmem_ld32f(to + (c_lo + cc) * 32, *reinterpret_cast<float(*)[32]>(&o[32 * cc]));
+    if (have) tc_wait_ld();
+    const int tile_row0 = rb * a.unit_rows + tile * kBM;  // first query row of the tile
+    const bool full_tile = nch == 1 && D == 128 && tile_row0 + kBM <= G * n && (tile == 0 || two);
+    if (nch > 1) {
+      char* sl = static_cast<char*>(a.ws) + a.slab_off + (size_t)slab * L::kSlabBytes;
+      uint4* sl8 = reinterpret_cast<uint4*>(sl);  // [D / 8][kRows] groups of 8 bf16
+      if (store) {
 #pragma unroll
         for (int cc = 0; cc < D / 32; ++cc) {
-          if (cc >= nch) break;
+          if (cc >= n32) break;
           const int c = c_lo + cc;
           const float* oc = &o[32 * cc];
-          uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c * 32);
 #pragma unroll
           for (int q = 0; q < 4; ++q)
-            dst[q] = live ? make_uint4(pack_bf16(oc[8 * q + 0] * inv, oc[8 * q + 1] * inv),
-                                       pack_bf16(oc[8 * q + 2] * inv, oc[8 * q + 3] * inv),
-                                       pack_bf16(oc[8 * q + 4] * inv, oc[8 * q + 5] * inv),
-                                       pack_bf16(oc[8 * q + 6] * inv, oc[8 * q + 7] * inv))
-                          : make_uint4(0u, 0u, 0u, 0u);
+            __stcg(sl8 + (c * 4 + q) * kRows + urw,
+                   live ? make_uint4(pack_bf16(oc[8 * q + 0] * inv, oc[8 * q + 1] * inv),
+                                     pack_bf16(oc[8 * q + 2] * inv, oc[8 * q + 3] * inv),
+                                     pack_bf16(oc[8 * q + 4] * inv, oc[8 * q + 5] * inv),
+                                     pack_bf16(oc[8 * q + 6] * inv, oc[8 * q + 7] * inv))
+                        : make_uint4(0u, 0u, 0u, 0u));
+        }
+        if (c_lo == 0) {
+          __stcg(reinterpret_cast<float*>(sl + L::kSlabM) + urw, live ? m_out * sl2 : NEG_INF);
+          __stcg(reinterpret_cast<float*>(sl + L::kSlabL) + urw, live ? l_out : 0.f);
         }
       }
-      if (store && c_lo == 0 && a.lse_out)
-        a.lse_out[orow] = live ? (m_out * sl2 + log2f(l_out)) * kLn2 : NEG_INF;
+      __threadfence();  // this thread's partial rows reach L2 before the unit's ticket
+    } else if (full_tile) {
+      // group g stages into its own buffer: tile 1's group uses V stage 0,
+      // the other (and, with one tile, both groups' regions) K stage 0
+      const uint32_t stage = (two ? (g == 0 ? k_base : v_base) : k_base);
+#pragma unroll
+      for (int cc = 0; cc < D / 32; ++cc) {
+        if (cc >= n32) break;
+        const int c = c_lo + cc;                  // 32-column chunk
+        const uint32_t region = stage + (uint32_t)((c >> 1) * kRegion) + (uint32_t)r * 128u;
+        const float* oc = &o[32 * cc];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int j = (c & 1) * 4 + q;          // 16-byte chunk within the 128-byte row
+          const uint4 v4 = make_uint4(pack_bf16(oc[8 * q + 0] * inv, oc[8 * q + 1] * inv),
+                                      pack_bf16(oc[8 * q + 2] * inv, oc[8 * q + 3] * inv),
+                                      pack_bf16(oc[8 * q + 4] * inv, oc[8 * q + 5] * inv),
+                                      pack_bf16(oc[8 * q + 6] * inv, oc[8 * q + 7] * inv));
+          st_shared_v4(region + (uint32_t)(((j ^ (r & 7)) << 4)), live ? v4 : make_uint4(0u, 0u, 0u, 0u));
+        }
+      }
+      fence_proxy_async_smem();  // generic stores -> bulk copy engine
+      group_bar(g);
+      if (r == 0) {
+        const int node0 = off + tile_row0 / G;
+        for (int c2 = c_lo / 2; c2 < (c_hi + 1) / 2; ++c2)
+          tma_store_3d(&tm_o, stage + (uint32_t)(c2 * kRegion), c2 * 64, h * G, node0);
+        bulk_commit();
+        bulk_wait_read0();  // the staging buffer is read before the CTA moves on
+      }
+    } else if (store) {
+#pragma unroll
+      for (int cc = 0; cc < D / 32; ++cc) {
+        if (cc >= n32) break;
+        const int c = c_lo + cc;
+        const float* oc = &o[32 * cc];
+        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c * 32);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          dst[q] = live ? make_uint4(pack_bf16(oc[8 * q + 0] * inv, oc[8 * q + 1] * inv),
+                                     pack_bf16(oc[8 * q + 2] * inv, oc[8 * q + 3] * inv),
+                                     pack_bf16(oc[8 * q + 4] * inv, oc[8 * q + 5] * inv),
+                                     pack_bf16(oc[8 * q + 6] * inv, oc[8 * q + 7] * inv))
+                        : make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    if (nch == 1 && store && c_lo == 0 && a.lse_out)
+      a.lse_out[orow] = live ? (m_out * sl2 + log2f(l_out)) * kLn2 : NEG_INF;
   }
   if (tid == 0) {
     // speculative K/V and Q copies this CTA did not consume land in buffers
@@ -751,6 +898,28 @@ __global__ void __maxnreg__(168)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
+  if (nch == 1) return;
+  // ---- a chunk of a split unit: the last of its nch chunks to finish
+  // merges them (no chunk ever waits for another).  Thread 0 publishes this
+  // CTA's partial rows (fence after the block barrier, then a ticket); the
+  // one that draws the unit's last ticket reads every chunk's rows.
+  int* misc_last = misc + 10;
+  if (tid == 0) {
+    int* ticket = static_cast<int*>(a.ws) + ((size_t)(b * a.Hkv + h) * a.rblocks + rb);
+    __threadfence();
+    const int t = atomicAdd(ticket, 1);
+    const bool last = t == nch - 1;
+    if (last) {
+      __threadfence();
+      atomicExch(ticket, 0);  // ready for the next launch
+    }
+    *misc_last = last ? 1 : 0;
+  }
+  __syncthreads();
+  if (*misc_last == 0) return;
+  const char* slabs = static_cast<const char*>(a.ws) + a.slab_off +
+                      (size_t)(slab - chunk) * L::kSlabBytes;
+  merge_chunks<D>(slabs, nch, rows, rb, G, n, off, h, a);
 }
 
 template <int D>
@@ -760,9 +929,12 @@ cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtenso
   auto kern = tree_attn_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc);
   if (e != cudaSuccess) return e;
+  // with key chunks (a workspace is given) a unit may become several items:
+  // at most `resident` more than the units in all
   const long long units = (long long)a.B * a.Hkv * a.rblocks;
+  const long long items = units + ((a.lpt && a.ws) ? a.resident : 0);
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)units, 1, 1);
+  cfg.gridDim = dim3((unsigned)items, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = L::kAlloc;
   cfg.stream = s;
@@ -805,13 +977,7 @@ int tree_attn_rblocks(int G, int max_nodes, int unit_rows) {
 // query tiles hold rows).  Occupancy is cached per device and head size.
 WholePlan tree_attn_whole_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max,
                                int num_sms) {
-  static int bps_cache[64][2] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
-  const int di = D == 64 ? 0 : 1;
-  int& bps = bps_cache[dev][di];
-  if (bps == 0) bps = di ? blocks_per_sm_d<128>() : blocks_per_sm_d<64>();
-  const long long resident = (long long)(bps > 0 ? bps : 1) * num_sms;
+  const long long resident = tree_attn_whole_resident(D, num_sms);
   const int tiles = (S_max + kBN - 1) / kBN;
   const double kFixed = 5.0;
   WholePlan best{kRows, B > 1 ? 1 : 0, 1e30};
@@ -823,6 +989,27 @@ WholePlan tree_attn_whole_plan(int D, int B, int Hkv, int G, int max_nodes, int 
     if (cost < best.cost_us - 1e-9) best = WholePlan{ur, B > 1 ? 1 : 0, cost};
   }
   return best;
+}
+
+int tree_attn_whole_resident(int D, int num_sms) {
+  static int bps_cache[64][2] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
+  const int di = D == 64 ? 0 : 1;
+  int& bps = bps_cache[dev][di];
+  if (bps == 0) bps = di ? blocks_per_sm_d<128>() : blocks_per_sm_d<64>();
+  return std::min((bps > 0 ? bps : 1) * num_sms, kWholeMaxResident);
+}
+
+// the tickets cover every unit id (b, h, rb) at the smaller unit size
+size_t tree_attn_whole_slab_off(int B, int Hkv, int G, int max_nodes) {
+  const long long units = (long long)B * Hkv * tree_attn_rblocks(G, max_nodes, kBM);
+  return (size_t)((units * 4 + 255) / 256 * 256);
+}
+
+size_t tree_attn_whole_ws_bytes(int D, int B, int Hkv, int G, int max_nodes) {
+  const size_t slab = D == 64 ? (size_t)Layout<64>::kSlabBytes : (size_t)Layout<128>::kSlabBytes;
+  return tree_attn_whole_slab_off(B, Hkv, G, max_nodes) + (size_t)2 * kWholeMaxResident * slab;
 }
 
 cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,

@@ -43,10 +43,18 @@ def test_status_strings(lib):
 
 
 def test_tree_attn_workspace_size(lib):
-    # two int counters per (tree, kv-head, 128-row work item) padded to 256 bytes, then
-    # per (work item, split) a slab of 128 rows x (D bf16 + 2 fp32), up to 10 splits
-    units = 1 * 8 * 2
-    assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 128) == 256 + units * 10 * 128 * 264
+    # The larger of the two kernels' needs.  Split kernel: two int counters per
+    # (tree, kv-head, 128-row work item) padded to 256 bytes, then per (work item,
+    # split) a slab of 128 rows x (D bf16 + 2 fp32), up to 10 splits.  Two-tile
+    # kernel: one ticket per 128-row unit padded to 256 bytes, then 512 slabs of
+    # 256 rows for the key chunks of long units (twice the 256 resident CTAs).
+    def sizes(B, n, Hq, Hkv, D):
+        units = B * Hkv * (((Hq // Hkv) * n + 127) // 128)
+        split = (units * 8 + 255) // 256 * 256 + units * 10 * 128 * (2 * D + 8)
+        whole = (units * 4 + 255) // 256 * 256 + 512 * 256 * (2 * D + 8)
+        return max(split, whole)
+    for args in ((1, 60, 32, 8, 128), (4, 128, 64, 8, 128), (64, 256, 32, 8, 128), (1, 16, 8, 8, 64)):
+        assert lib.treegraft_tree_attn_workspace_size(*args) == sizes(*args), args
     assert lib.treegraft_tree_attn_workspace_size(1, 60, 32, 8, 96) == 0
 
 
