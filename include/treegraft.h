@@ -250,8 +250,9 @@ int treegraft_graft_expand(const void* logits, int dtype, int logit_rows, int V,
  * path int32 [B, path_cap] (path_cap >= 1); accept_len, bonus int32 [B].
  * ws       scratch of treegraft_accept_workspace_size(B, n_total) bytes,
  *          16-byte aligned, ZERO-FILLED before its first use with this
- *          function; each call leaves it ready for the next call.  Calls
- *          sharing one ws must not overlap on the GPU.
+ *          function; each call on well-formed trees leaves it all zero
+ *          again, so one ws serves later calls of any B and n_total that
+ *          fit it.  Calls sharing one ws must not overlap on the GPU.
  * Errors: TG_ERR_INVALID_ARG, TG_ERR_UNSUPPORTED (V > 262144 for bf16 or
  *   > 131072 for fp32), TG_ERR_CUDA;
  *   a malformed tree sets TG_ERR_DEVICE_TREE, a path longer than path_cap
@@ -418,8 +419,10 @@ int treegraft_grow_step(int mode, const void* logits, int dtype, int V, int64_t 
  * device, drawn by the caller (u[c, 0] decides child c, u[v, 1] the bonus
  * draw at v).  temperature > 0 (fp32 must be able to hold log2(e) / T).
  * ws: treegraft_accept_sample_workspace_size(B, n_total) bytes, 16-byte
- * aligned, ZEROED before its first use (per-tree tickets, reset by every
- * call).  One launch: per node row, the masses 2^((l - max) log2(e) / T)
+ * aligned, ZEROED before its first use (per-node flags and candidates,
+ * per-tree tickets); each call on well-formed input leaves it all zero
+ * again, so one ws serves later calls of any B and n_total that fit it.
+ * One launch: per node row, the masses 2^((l - max) log2(e) / T)
  * in 44-bit fixed point (exact, order-free sums), every child's decision
  * and the bonus draw the row would give if the walk ended there; the CTA
  * that finishes a tree's rows walks it.  The masses carry the rounding of

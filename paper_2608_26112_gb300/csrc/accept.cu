@@ -9,8 +9,9 @@
 //   ok[v]   = token[v] == am[pa(v)]
 //   full[v] = AND of ok over the root..v chain, depth[v] = its length
 //   a*      = argmax over full nodes of (depth, -id)
-// then writes the root..a* path, A = depth(a*) and the bonus token am[a*],
-// and resets the ticket so the scratch is ready for the next call.
+// then writes the root..a* path, A = depth(a*) and the bonus token am[a*].
+// The walker returns the ticket and the tree's argmax slots to zero, so the
+// scratch is all zero again for the next call, whatever its shape.
 // Every node's row is scanned because the bonus token needs the row of a*,
 // which may be any node (a leaf included).
 #include <cooperative_groups.h>
@@ -105,13 +106,13 @@ __global__ void __launch_bounds__(kScanThreads, 4) accept_kernel(AcceptArgs a, i
   if (tid == 0) {
     uint64_t best = 0;
     for (int c = 0; c < C; ++c) best = sm.recv_key[c] > best ? sm.recv_key[c] : best;
-    a.am[row] = (int32_t)key_index(best);
-    // release: the argmax store above is visible to the CTA that draws the
+    // release: the argmax store below is visible to the CTA that draws the
     // last ticket; acquire: the last CTA sees every other row's argmax
     if (bad_tree) {
-      sm.last = 0;  // a malformed extent never touches the ticket
+      sm.last = 0;  // a row in no tree stores nothing and never touches a ticket
       raise_status(a.status, kStTree);
     } else {
+      a.am[row] = (int32_t)key_index(best);
       const int t = atom_add_acq_rel_gpu(&a.tickets[b], 1);
       sm.last = (t == n - 1);
       if (sm.last) a.tickets[b] = 0;  // ready for the next call (the next launch orders it)
@@ -123,7 +124,10 @@ __global__ void __launch_bounds__(kScanThreads, 4) accept_kernel(AcceptArgs a, i
   if (!sm.last) return;
 
   // ---- walk of tree b (this CTA saw every row of the tree finish)
-  if (tid < n) sm.am[tid] = __ldcg(&a.am[off + tid]);
+  if (tid < n) {
+    sm.am[tid] = __ldcg(&a.am[off + tid]);
+    a.am[off + tid] = 0;
+  }
   const bool bad = (tid < n) && (tid == 0 ? (v_par != -1) : (v_par < 0 || v_par >= tid));
   if (__syncthreads_or(bad)) {
     if (tid == 0) raise_status(a.status, kStTree);

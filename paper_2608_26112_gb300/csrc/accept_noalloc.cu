@@ -30,7 +30,7 @@ constexpr int kNoAllocMaxNodes = TG_NOALLOC_MAX_NODES;
 constexpr int kNoAllocMaxTrees = TG_NOALLOC_MAX_TREES;
 constexpr int kNoAllocScratchWords = kNoAllocMaxNodes + kNoAllocMaxTrees;
 
-// argmax per node in [0, kNoAllocMaxNodes), ticket counters after it
+// a call's B ticket counters, then the argmax slots of its n_total nodes
 static __device__ __align__(256) int32_t g_accept_scratch[kNoAllocScratchWords];
 
 constexpr int kMaxDevices = 64;
@@ -75,9 +75,10 @@ extern "C" int treegraft_accept_noalloc(const void* target_logits, int dtype, in
   int32_t* scratch = scratch_ptr();
   if (!st || !scratch) return TG_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // the ticket counters must start at zero; the array keeps whatever the
-  // previous call left, so clear them on the stream before the launch
-  if (cudaMemsetAsync(scratch + kNoAllocMaxNodes, 0, sizeof(int32_t) * (size_t)B, s) != cudaSuccess)
+  // the tickets and argmax slots must start at zero; a well-formed call
+  // leaves them so, but the array keeps whatever a malformed one left, so
+  // clear them (tickets [0, B), slots [B, B + n_total)) before the launch
+  if (cudaMemsetAsync(scratch, 0, sizeof(int32_t) * ((size_t)B + (size_t)n_total), s) != cudaSuccess)
     return TG_ERR_CUDA;
   AcceptArgs a;
   a.logits = target_logits;
@@ -93,8 +94,8 @@ extern "C" int treegraft_accept_noalloc(const void* target_logits, int dtype, in
   a.path = path;
   a.accept_len = accept_len;
   a.bonus = bonus;
-  a.am = scratch;
-  a.tickets = scratch + kNoAllocMaxNodes;
+  a.tickets = scratch;
+  a.am = scratch + B;
   a.status = st;
   return launch_accept(a, s) == cudaSuccess ? TG_OK : TG_ERR_CUDA;
 }

@@ -316,6 +316,14 @@ __global__ void __launch_bounds__(kScanThreads, 4) sample_kernel(SampleArgs a, i
   __syncthreads();
   if (!sm.last) return;
 
+  // this tree's flags and candidates; their slots go back to zero, so that
+  // with the ticket the whole workspace is zero again for the next call
+  const int f = (tid > 0 && tid < n) ? __ldcg(a.flag + off + tid) : 0;
+  const int cand = tid < n ? __ldcg(a.bcand + off + tid) : 0;
+  if (tid < n) {
+    a.flag[off + tid] = 0;
+    a.bcand[off + tid] = 0;
+  }
   // ---- walk of tree b along the first accepted child of every node
   const bool bad = (tid < n) && (tid == 0 ? (v_par != -1) : (v_par < 0 || v_par >= tid));
   if (__syncthreads_or(bad)) {
@@ -323,8 +331,7 @@ __global__ void __launch_bounds__(kScanThreads, 4) sample_kernel(SampleArgs a, i
     return;
   }
   sm.next[tid] = 0x7FFFFFFF;
-  const int f = (tid > 0 && tid < n) ? __ldcg(a.flag + off + tid) : 0;
-  if (tid < n) sm.tok[tid] = __ldcg(a.bcand + off + tid);  // the tokens are not needed any more
+  if (tid < n) sm.tok[tid] = cand;  // the tokens are not needed any more
   __syncthreads();
   if (f) atomicMin(&sm.next[v_par], tid);
   __syncthreads();

@@ -380,6 +380,33 @@ def test_accept_rows_outside_every_tree_set_status(dev, where):
         np.testing.assert_array_equal(g.cpu().numpy(), r)
 
 
+def test_accept_one_workspace_serves_any_shape(dev):
+    """The walk returns every ticket and argmax slot of a well-formed call to
+    zero, even when the tree's path does not fit path_cap, so one workspace
+    sized for the largest call serves later calls of other B and n_total
+    (their tickets then sit where an earlier call kept argmax slots)."""
+    big = synth.make_workload("llama3-70b-verify", seed=31, with_strong=False)
+    ws = tg.accept_workspace(len(big["node_off"]) - 1, len(big["parent"]), dev)
+    for name, seed, cap in (("llama3-70b-verify", 31, None), ("tiny", 32, 2),
+                            ("llama3-8b-verify", 33, None), ("tiny", 34, None)):
+        wl = synth.make_workload(name, seed=seed, with_strong=False)
+        bf = wl["logits"].dtype == np.uint16
+        full = _dev.max_nodes(wl)
+        got = tg.accept(_dev.logits(wl, dev), _dev.i32(wl["token"], dev),
+                        _dev.i32(wl["parent"], dev), _dev.i32(wl["node_off"], dev), full,
+                        cap or full, ws)
+        st = tg.last_device_status()
+        assert not torch.any(ws != 0)
+        if cap is None:
+            assert st == 0
+            ref = O.accept(wl["logits"], wl["token"], wl["parent"], wl["node_off"], full, bf16=bf)
+            for g, r in zip(got, ref):
+                np.testing.assert_array_equal(g.cpu().numpy(), r)
+        else:
+            ref = O.accept(wl["logits"], wl["token"], wl["parent"], wl["node_off"], full, bf16=bf)
+            assert (st & 16) == (16 if ref[1].max() + 1 > cap else 0)
+
+
 def test_accept_grafting_examples(dev):
     import json, os
     with open(os.path.join(os.path.dirname(__file__), "golden", "grafting_examples.json")) as f:
@@ -560,6 +587,51 @@ def test_tree_attn_serving_sweep(dev, B):
         count = int(wl["prefix_len"][b]) + O.node_depth(wl["parent"][a:e]) + 1
         np.testing.assert_allclose(lse[a:e], np.log(count)[:, None] * np.ones((1, sh["Hq"])),
                                    atol=LSE_ABS, rtol=0)
+
+
+def test_tree_attn_long_tree_cut_into_key_chunks(dev):
+    """One long tree among short ones: the batch runs as whole units dealt
+    longest first, and the long tree's units are cut into key chunks (about
+    one resident CTA's share of the batch each) whose last one to finish
+    merges them.  The long tree and a short one carry random K/V and are
+    checked against the oracle; the others have all-zero K/V (outputs exactly
+    0, lse = ln of the number of keys each node sees).  Two calls in a row on
+    the same workspace: the chunk tickets are back at zero after each."""
+    P = [8000, 300, 500, 700, 900, 1100, 1300, 1500, 1700]
+    n = [64, 40, 48, 56, 64, 72, 80, 88, 96]
+    shape = _attn_shape(len(P), P, n, [6] * len(P), 32, 8, 128, cap=10)
+    drawn = [0, 4]
+    wl = synth.make_workload(shape, seed=31, with_logits=False, with_strong=False, kv_trees=drawn)
+    k, v = _serving_kv(wl, dev)
+    q = _dev.bf16(wl["q"], dev)
+    sh = wl["shape"]
+    B = len(P)
+    ws = torch.zeros(tg.tree_attn_workspace_size(B, _dev.max_nodes(wl), 32, 8, 128),
+                     dtype=torch.uint8, device=dev)
+    off = wl["node_off"]
+    refs = {}
+    for i, b in enumerate(drawn):
+        a, e = int(off[b]), int(off[b + 1])
+        refs[b] = O.tree_attention(wl["q"][a:e], wl["k_cache"][i:i + 1], wl["v_cache"][i:i + 1],
+                                   wl["prefix_len"][b:b + 1], wl["parent"][a:e], [0, e - a], Hkv=8)
+    for _ in range(2):
+        lse = torch.full((q.shape[0], q.shape[1]), float("nan"), device=dev)
+        out, _ = tg.tree_attn(q, k, v, _dev.i32(wl["prefix_len"], dev), _dev.i32(wl["parent"], dev),
+                              _dev.i32(wl["node_off"], dev), _dev.max_nodes(wl), lse_out=lse, ws=ws)
+        _status_clean()
+        o = _dev.bf16_to_np(out)
+        lse = lse.cpu().numpy().astype(np.float64)
+        for b in drawn:
+            a, e = int(off[b]), int(off[b + 1])
+            _check_attn(wl, o[a:e], lse[a:e], *refs[b])
+        for b in range(B):
+            if b in drawn:
+                continue
+            a, e = int(off[b]), int(off[b + 1])
+            assert np.all(o[a:e] == 0.0)
+            count = int(wl["prefix_len"][b]) + O.node_depth(wl["parent"][a:e]) + 1
+            np.testing.assert_allclose(lse[a:e], np.log(count)[:, None] * np.ones((1, 32)),
+                                       atol=LSE_ABS, rtol=0)
 
 
 def test_accept_serving_sweep(dev):

@@ -73,6 +73,7 @@ def _run(dev, rng, sizes, V, bf16, T, cap=10, path_cap=12, dup_prob=0.0, bump=12
                                              _dev.f32(u, dev), T, ws)
         torch.cuda.synchronize()
         assert tg.last_device_status() == 0
+        assert not torch.any(ws != 0)       # flags, candidates and tickets back to zero
     path, alen, bonus = (t.cpu().numpy() for t in (path, alen, bonus))
     op, oa, ob, info = S.accept_sample(host, token, parent, off, u, T, path_cap, bf16=bf16)
     exact = 0
@@ -159,3 +160,27 @@ def test_sample_rejects_bad_temperature(dev):
     with pytest.raises(tg.TreeGraftError):
         tg.accept_sample(x, i, torch.tensor([-1, 0], dtype=torch.int32, device=dev), off, 2, 4,
                          u, 0.0, ws)
+
+
+def test_sample_one_workspace_serves_any_shape(dev):
+    """A workspace sized for a 24-tree batch serves a 3-tree batch next: its
+    tickets then sit where the first call kept per-node flags, which the walk
+    has returned to zero."""
+    rng = synth.make_rng(977)
+    sizes = rng.integers(20, 41, size=24).tolist()
+    parent, token, off = _trees(rng, sizes, 1024, 10)
+    ws = tg.accept_sample_workspace(len(sizes), len(parent), dev)
+    for sz in (sizes, [5, 9, 3]):
+        parent, token, off = _trees(rng, sz, 1024, 10)
+        host = _logits(rng, parent, token, off, 1024, False, bump=12.0)
+        u = rng.random((len(parent), 2)).astype(np.float32)
+        path, alen, bonus = tg.accept_sample(_dev.f32(host, dev), _dev.i32(token, dev),
+                                             _dev.i32(parent, dev), _dev.i32(off, dev), max(sz),
+                                             12, _dev.f32(u, dev), 1.0, ws)
+        torch.cuda.synchronize()
+        assert tg.last_device_status() == 0
+        assert not torch.any(ws != 0)
+        op, oa, ob, info = S.accept_sample(host, token, parent, off, u, 1.0, 12, bf16=False)
+        for b in range(len(sz)):
+            if info[b]["margin"] > MARGIN:
+                assert path[b].tolist() == op[b].tolist() and alen[b] == oa[b]
