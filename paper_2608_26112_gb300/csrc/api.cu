@@ -202,7 +202,11 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
   const int mtiles = (G * max_nodes + 127) / 128;
   double split_cost = 0.0;
   const SplitPlan sp = tree_attn_split_plan(D, B, Hkv, mtiles, S_max, nsm, &split_cost);
-  const WholePlan wp = tree_attn_whole_plan(D, B, Hkv, G, max_nodes, S_max, nsm);
+  // long units are cut into key chunks merged through the workspace when it
+  // is large enough; otherwise every unit stays whole
+  const bool chunks =
+      ws && aligned16(ws) && ws_bytes >= tree_attn_whole_ws_bytes(D, B, Hkv, G, max_nodes);
+  const WholePlan wp = tree_attn_whole_plan(D, B, Hkv, G, max_nodes, S_max, nsm, chunks);
   const cudaStream_t cs = static_cast<cudaStream_t>(stream);
   // With a wave of work items or more there is nothing to split: whole
   // units in longest-first order (ragged batches) are then the better plan.
@@ -211,9 +215,6 @@ int treegraft_tree_attn(const void* q, const void* k_cache, const void* v_cache,
     a.unit_rows = wp.unit_rows;
     a.rblocks = tree_attn_rblocks(G, max_nodes, wp.unit_rows);
     a.lpt = wp.lpt;
-    // long units are cut into key chunks merged through the workspace when
-    // it is large enough; otherwise every unit stays whole
-    const bool chunks = ws && aligned16(ws) && ws_bytes >= tree_attn_whole_ws_bytes(D, B, Hkv, G, max_nodes);
     a.ws = chunks ? ws : nullptr;
     a.slab_off = tree_attn_whole_slab_off(B, Hkv, G, max_nodes);
     a.resident = tree_attn_whole_resident(D, nsm);

@@ -40,7 +40,7 @@ cudaError_t launch_tree_attn(const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                              cudaStream_t s);
 int tree_attn_rblocks(int G, int max_nodes, int unit_rows);
 WholePlan tree_attn_whole_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max,
-                               int num_sms);
+                               int num_sms, bool chunks);
 // workspace of the two-tile kernel: unit tickets, then the partial-row slabs
 // of the key chunks (at most kWholeMaxSlabs, twice the resident CTAs)
 size_t tree_attn_whole_ws_bytes(int D, int B, int Hkv, int G, int max_nodes);

@@ -37,6 +37,7 @@
 // from prefix_len and node_off), so ragged batches end together.
 // Every mbarrier wait is bounded.
 #include <algorithm>
+#include <cmath>
 
 #include "common.cuh"
 #include "launch.h"
@@ -972,21 +973,37 @@ int tree_attn_rblocks(int G, int max_nodes, int unit_rows) {
 
 // Whole-unit plan for this kernel: units of 256 rows (two query tiles
 // sharing each K/V tile) or of 128 rows, and the estimated launch time
-// (microseconds, fitted to measured launches): waves of resident CTAs, each
-// a fixed part plus one part per 128-key tile of its unit (larger when both
-// query tiles hold rows).  Occupancy is cached per device and head size.
+// (microseconds, fitted to measured launches).  A 128-key tile costs about
+// the same with one query tile as with two (the chain S -> softmax -> PV of
+// a tile sets the pace, and two tiles overlap theirs), so 256-row units do
+// twice the work per CTA.  Without key chunks: waves of resident CTAs, each
+// a fixed part plus one part per key tile of its unit.  With key chunks (a
+// batch with a large enough workspace), the longest-first list spreads the
+// tiles over the resident CTAs: the longer of the average share and the
+// longest item, a fixed part per item of a CTA, and a merge when units are
+// cut.  Occupancy is cached per device and head size.
 WholePlan tree_attn_whole_plan(int D, int B, int Hkv, int G, int max_nodes, int S_max,
-                               int num_sms) {
+                               int num_sms, bool chunks) {
   const long long resident = tree_attn_whole_resident(D, num_sms);
   const int tiles = (S_max + kBN - 1) / kBN;
-  const double kFixed = 5.0;
-  WholePlan best{kRows, B > 1 ? 1 : 0, 1e30};
+  const double kFixed = 5.0, kMerge = 2.0;
+  const int lpt = B > 1 ? 1 : 0;
+  WholePlan best{kRows, lpt, 1e30};
   for (int ur = kRows; ur >= kBM; ur -= kBM) {
     const long long units = (long long)B * Hkv * tree_attn_rblocks(G, max_nodes, ur);
     const int rows = std::min(ur, G * max_nodes);
-    const double per_tile = rows > kBM ? 1.8 : 1.0;
-    const double cost = (double)((units + resident - 1) / resident) * (kFixed + per_tile * tiles);
-    if (cost < best.cost_us - 1e-9) best = WholePlan{ur, B > 1 ? 1 : 0, cost};
+    const double per_tile = rows > kBM ? 1.9 : 1.85;
+    double cost = (double)((units + resident - 1) / resident) * (kFixed + per_tile * tiles);
+    if (lpt && chunks) {
+      // average tiles per CTA, the longest item (a chunk or a whole unit),
+      // the items each CTA runs
+      const double avg = (double)units * tiles / (double)resident;
+      const double len = std::min((double)tiles, std::max((double)kWholeChunkMin, std::ceil(1.25 * avg)));
+      const double nch = std::ceil((double)tiles / len);
+      const double per_cta = std::ceil((double)units * nch / (double)resident);
+      cost = std::min(cost, per_cta * kFixed + (nch > 1 ? kMerge : 0.0) + per_tile * std::max(len, avg));
+    }
+    if (cost < best.cost_us - 1e-9) best = WholePlan{ur, lpt, cost};
   }
   return best;
 }
