@@ -80,15 +80,21 @@ typedef enum { TG_BF16 = 0, TG_F32 = 1 } tg_dtype;
  * scale    softmax scale; 0 selects D^-1/2.
  * out      bf16 [n_total, Hq, D];  lse_out fp32 [n_total, Hq] or NULL.
  * ws       scratch of treegraft_tree_attn_workspace_size(B, max_nodes, Hq,
- *          Hkv, D) bytes, 16-byte aligned, ZERO-FILLED before its first use:
- *          split counters (returned to zero by every call) and the partial
- *          rows of the split-KV combine.  Calls sharing one ws must not
- *          overlap on the GPU.  Small problems split the keys of a work
- *          unit over several thread blocks of a cooperative launch (the
- *          whole grid resident at once) that meet on those counters (a
- *          bounded wait, see treegraft_set_wait_budget: TG_ERR_TIMEOUT,
- *          never a hang).  The size is 0 when these sizes never split; ws
- *          may then be NULL.
+ *          Hkv, D) bytes, 16-byte aligned, ZERO-FILLED before its first use;
+ *          every call returns its counters to zero.  Calls sharing one ws
+ *          must not overlap on the GPU.  Two plans use it:
+ *          - small problems split the keys of a 128-row work unit over
+ *            several thread blocks of a cooperative launch (the whole grid
+ *            resident at once) that meet on counters in ws (a bounded wait,
+ *            see treegraft_set_wait_budget: TG_ERR_TIMEOUT, never a hang)
+ *            and combine their partial rows through ws;
+ *          - batches whose whole units fill the GPU cut the keys of units
+ *            well above the average share into chunks; each chunk writes
+ *            its partial rows to ws and the last chunk of a unit to finish
+ *            (a ticket in ws, no waiting) merges them.
+ *          ws may be NULL (ws_bytes 0) when the sizes fill the GPU with
+ *          whole units: every unit then stays whole.  A small problem
+ *          without enough ws returns TG_ERR_INVALID_ARG.
  * Errors: TG_ERR_INVALID_ARG (null pointer, bad sizes, misaligned q/k/v),
  *   TG_ERR_UNSUPPORTED (D or G outside the list), TG_ERR_CUDA.  A malformed
  *   tree sets TG_ERR_DEVICE_TREE; its rows of `out` and `lse_out` are then
