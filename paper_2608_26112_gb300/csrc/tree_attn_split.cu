@@ -267,7 +267,7 @@ __device__ __forceinline__ void combine_rows(const char* slabs, int split, int r
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
-    tree_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
+    tree_attn_split_kernel(const __grid_constant__ CUtensorMap tm_q,
                      const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const AttnArgs a) {
   using L = Layout<D>;
@@ -772,7 +772,7 @@ template <int D>
 cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                      const AttnArgs& a, SplitPlan plan, cudaStream_t s) {
   using L = Layout<D>;
-  auto kern = tree_attn_kernel<D>;
+  auto kern = tree_attn_split_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc);
   if (e != cudaSuccess) return e;
   const int G = a.Hq / a.Hkv;
@@ -805,7 +805,7 @@ cudaError_t launch_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtenso
 template <int D>
 int max_active_clusters_d(int splits) {
   using L = Layout<D>;
-  auto kern = tree_attn_kernel<D>;
+  auto kern = tree_attn_split_kernel<D>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc) !=
       cudaSuccess)
     return 0;
@@ -832,7 +832,7 @@ int max_active_clusters_d(int splits) {
 template <int D>
 int blocks_per_sm_d() {
   using L = Layout<D>;
-  auto kern = tree_attn_kernel<D>;
+  auto kern = tree_attn_split_kernel<D>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kAlloc) !=
       cudaSuccess)
     return 0;
