@@ -848,11 +848,15 @@ int blocks_per_sm_d() {
 
 // How to split the keys.  Cost model: waves of resident work items times
 // the per-CTA time, a fixed part plus one part per 128-key tile of its
-// split.  A cluster path holds up to 8 splits, with the resident clusters
-// per split count from the occupancy API; a cooperative path holds up to
-// kAttnMaxSplits when the whole grid is resident at once (one wave).  On a
-// tie the cluster path wins (no counters).  Occupancy figures are cached
-// per device and head size.
+// split, plus the combine when the keys are split.  The constants are fitted
+// to a measured timeline of the Llama-3-8B-shaped launch (9 splits of 17
+// key tiles): launch to first S product 3.5 us, 1.05 us per key tile, and
+// 4.7 us from the last product to the merged rows (partials through L2, the
+// counter barrier, the merge).  A cluster path holds up to 8 splits, with
+// the resident clusters per split count from the occupancy API; a
+// cooperative path holds up to kAttnMaxSplits when the whole grid is
+// resident at once (one wave).  On a tie the cluster path wins (no
+// counters).  Occupancy figures are cached per device and head size.
 SplitPlan tree_attn_split_plan(int D, int B, int Hkv, int mtiles, int S_max, int num_sms,
                                 double* cost_us) {
   static int cache[64][2][kClusterMaxSplits + 1] = {};
@@ -862,7 +866,7 @@ SplitPlan tree_attn_split_plan(int D, int B, int Hkv, int mtiles, int S_max, int
   const int di = D == 64 ? 0 : 1;
   const long long units = (long long)B * Hkv * mtiles;
   const int tiles = (S_max + kBN - 1) / kBN;
-  const double kFixed = 5.0, kCombine = 1.0, kPerTile = 0.9;  // microseconds, measured scale
+  const double kFixed = 3.5, kCombine = 4.7, kPerTile = 1.05;  // microseconds
   int& bps = bps_cache[dev][di];
   if (bps == 0) bps = di ? blocks_per_sm_d<128>() : blocks_per_sm_d<64>();
   const long long coop_cap = (long long)(bps > 0 ? bps : 1) * num_sms;
