@@ -640,7 +640,7 @@ def grow_timing(seed, dev, stream, reps, n_sets=3):
     b = rows * V * 2
     return {"us": t * 1e6, "schedule": GROW_SCHEDULE, "W": W, "m": m, "vocab": V,
             "nodes_out": cap, "rows_scanned": rows, "bytes": b, "GBps": b / t / 1e9,
-            "launches": 3 * len(GROW_SCHEDULE), "in_step": False,
+            "launches": 2 * len(GROW_SCHEDULE), "in_step": False,
             "note": "Algorithm 2 grow loop; bytes = drafter-table rows scanned x V x 2"}
 
 
@@ -741,7 +741,7 @@ def ngram_timing(seed, dev, stream, reps, n_sets=3):
         loops = max(5, reps // 10)
         t = time_graph(g, loops, stream) / (loops * n_sets)
         out[label] = {"schedule": schedule, "W": W, "m": m, "nodes_out": cap, "us": t * 1e6,
-                      "launches": sum(3 if a == 1 else 1 for a in schedule)}
+                      "launches": sum(2 if a == 1 else 1 for a in schedule)}
     return out
 
 
