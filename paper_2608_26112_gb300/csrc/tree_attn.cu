@@ -93,6 +93,9 @@ struct Layout {
   static constexpr int kSlabBytes = kRows * (2 * D + 8);
   static constexpr int kSlabM = kRows * D * 2;
   static constexpr int kSlabL = kSlabM + kRows * 4;
+  // chunks of one unit: the merge keeps two floats per (chunk, row) over the
+  // tile buffers
+  static constexpr int kMaxChunks = kTileEnd / (kRows * 8);
 };
 
 // 32 mask bits of one node for tree slots [b0, b0 + 32): slot < 0 is the
@@ -170,15 +173,16 @@ __device__ __forceinline__ void group_bar(int g) {
 // The work item this CTA computes in a longest-first launch.  Every CTA
 // derives the same list from prefix_len and node_off: the total work W (key
 // tiles summed over units), a chunk length L = max(chunk_min, ceil(1.25 W /
-// resident CTAs)), and for each tree nch = ceil(tiles / L) key chunks per
-// unit (a unit whose keys are split this way has its chunks merged by the
-// last one to finish).  Trees are ranked by chunk length (desc, tree id asc),
+// resident CTAs)), and for each tree nch = min(max_chunks, ceil(tiles / L))
+// key chunks per unit (a unit whose keys are split this way has its chunks
+// merged by the last one to finish).  Trees are ranked by chunk length (desc, tree id asc),
 // items of a tree by (kv-head, row block, chunk); the slot-th item of that
 // order is this CTA's.  All threads take part; the result goes to misc:
 // [0] b (-1 past the last item), [1] h, [2] rb, [3] chunk, [6] chunks of the
 // unit, [7] partial-row slab of the item (-1 for a whole unit).  Invalid
 // tree extents count as one item of length 0 (its CTA raises the status).
-__device__ void lpt_item(const AttnArgs& a, int G, long long slot, int* scratch, int* misc) {
+__device__ void lpt_item(const AttnArgs& a, int G, long long slot, int max_chunks, int* scratch,
+                         int* misc) {
   const int B = a.B;
   int* tiles = scratch;
   int* units = scratch + B;
@@ -207,7 +211,7 @@ __device__ void lpt_item(const AttnArgs& a, int G, long long slot, int* scratch,
       a.ws ? max((long long)a.chunk_min, (5 * *wsum + 4ll * a.resident - 1) / (4ll * a.resident))
            : (1ll << 40);
   for (int t = threadIdx.x; t < B; t += kThreads)
-    nch[t] = tiles[t] > 0 ? (int)((tiles[t] + chunk - 1) / chunk) : 1;
+    nch[t] = tiles[t] > 0 ? (int)min((long long)max_chunks, (tiles[t] + chunk - 1) / chunk) : 1;
   __syncthreads();
   for (int t = threadIdx.x; t < B; t += kThreads) {
     const int mine = (tiles[t] + nch[t] - 1) / nch[t];
@@ -284,67 +288,87 @@ __device__ void lpt_item(const AttnArgs& a, int G, long long slot, int* scratch,
 // (Sec. 3.1 attention as a softmax over the union of the chunks' keys).
 // Chunk s holds O_s / l_s (bf16), its max m_s (base 2) and sum l_s: with
 // w_s = 2^(m_s - M) l_s, M = max_s m_s, the row is o = sum_s w_s (O_s / l_s)
-// / sum_s w_s and lse = ln 2 (M + log2 sum_s w_s).  Every thread of the CTA
-// takes (row, 8-column group) items; a batch's loads are all in flight at
-// once.
+// / sum_s w_s and lse = ln 2 (M + log2 sum_s w_s).  First one thread per
+// row turns the chunks' (m_s, l_s) into normalised weights in shared memory
+// (`wgt`, nc x kRows floats over the CTA's idle tile buffers); then every
+// thread accumulates kU (row, 8-column group) items at a time, the loads of
+// all kU items of a chunk in flight together, so the merge costs a few L2
+// round trips per chunk rather than one per item.  Kept out of line:
+// inlined, its registers made the kernel spill.
 template <int D>
-__device__ void merge_chunks(const char* slabs, int nc, int rows, int rb, int G, int n, int off,
-                             int h, const AttnArgs& a) {
+__device__ __noinline__ void merge_chunks(const char* slabs, int nc, int rows, int rb, int G, int n,
+                                          int off, int h, float* wgt, const AttnArgs& a) {
   using L = Layout<D>;
   const float NEG_INF = __int_as_float(0xff800000);
   constexpr int CG = D / 8;
-  constexpr int kBatch = 8;
-  for (int item = threadIdx.x; item < rows * CG; item += kThreads) {
-    const int ur = item % rows, c8 = item / rows;  // row-fastest: coalesced slab reads
+  constexpr int kU = 4;
+  for (int ur = threadIdx.x; ur < rows; ur += kThreads) {
+    float M = NEG_INF;
+    for (int s = 0; s < nc; ++s) {
+      const float m = __ldcg(reinterpret_cast<const float*>(slabs + (size_t)s * L::kSlabBytes +
+                                                            L::kSlabM) + ur);
+      const float l = __ldcg(reinterpret_cast<const float*>(slabs + (size_t)s * L::kSlabBytes +
+                                                            L::kSlabL) + ur);
+      wgt[s * kRows + ur] = m;  // m and l parked, weighted below
+      wgt[(nc + s) * kRows + ur] = l;
+      M = fmaxf(M, m);
+    }
+    float Ls = 0.f;
+    for (int s = 0; s < nc; ++s) {
+      const float m = wgt[s * kRows + ur];
+      const float w = (m == NEG_INF) ? 0.f : ex2(m - M) * wgt[(nc + s) * kRows + ur];
+      wgt[s * kRows + ur] = w;
+      Ls += w;
+    }
+    const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
+    for (int s = 0; s < nc; ++s) wgt[s * kRows + ur] *= inv;
     const int rg = rb * a.unit_rows + ur;
     const int uu = rg / G, g = rg % G;
-    if (uu >= n) continue;
-    float M = NEG_INF, Ls = 0.f;
-    float acc[8];
+    if (uu < n && a.lse_out)
+      a.lse_out[(size_t)(off + uu) * a.Hq + (size_t)(h * G + g)] =
+          (M == NEG_INF || !(Ls > 0.f)) ? NEG_INF : (M + log2f(Ls)) * kLn2;
+  }
+  __syncthreads();
+  const int total = rows * CG;
+  for (int base = threadIdx.x; base < total; base += kU * kThreads) {
+    float acc[kU][8];
 #pragma unroll
-    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-    for (int s0 = 0; s0 < nc; s0 += kBatch) {
-      float mv[kBatch], lv[kBatch];
-      uint4 ov[kBatch];
+    for (int u = 0; u < kU; ++u)
 #pragma unroll
-      for (int j = 0; j < kBatch; ++j) {
-        const char* src = slabs + (size_t)min(s0 + j, nc - 1) * L::kSlabBytes;
-        mv[j] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabM) + ur);
-        lv[j] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabL) + ur);
-        ov[j] = __ldcg(reinterpret_cast<const uint4*>(src) + (size_t)c8 * kRows + ur);
+      for (int q = 0; q < 8; ++q) acc[u][q] = 0.f;
+    for (int s = 0; s < nc; ++s) {
+      const uint4* o = reinterpret_cast<const uint4*>(slabs + (size_t)s * L::kSlabBytes);
+      uint4 ov[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int item = min(base + u * kThreads, total - 1);
+        ov[u] = __ldcg(o + (size_t)(item / rows) * kRows + item % rows);  // row-fastest
       }
 #pragma unroll
-      for (int j = 0; j < kBatch; ++j)
-        if (s0 + j >= nc) mv[j] = NEG_INF;
-      float Mb = M;
-#pragma unroll
-      for (int j = 0; j < kBatch; ++j) Mb = fmaxf(Mb, mv[j]);
-      if (Mb == NEG_INF) continue;
-      if (Mb > M) {
-        const float cf = (M == NEG_INF) ? 0.f : ex2(M - Mb);
-        Ls *= cf;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) acc[q] *= cf;
-        M = Mb;
-      }
-#pragma unroll
-      for (int j = 0; j < kBatch; ++j) {
-        const float wt = (mv[j] == NEG_INF) ? 0.f : ex2(mv[j] - M) * lv[j];
-        Ls += wt;
-        const uint32_t wd[4] = {ov[j].x, ov[j].y, ov[j].z, ov[j].w};
+      for (int u = 0; u < kU; ++u) {
+        const int item = min(base + u * kThreads, total - 1);
+        const float w = wgt[s * kRows + item % rows];
+        const uint32_t wd[4] = {ov[u].x, ov[u].y, ov[u].z, ov[u].w};
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          acc[2 * q] = fmaf(wt, __uint_as_float(wd[q] << 16), acc[2 * q]);
-          acc[2 * q + 1] = fmaf(wt, __uint_as_float(wd[q] & 0xFFFF0000u), acc[2 * q + 1]);
+          acc[u][2 * q] = fmaf(w, __uint_as_float(wd[q] << 16), acc[u][2 * q]);
+          acc[u][2 * q + 1] = fmaf(w, __uint_as_float(wd[q] & 0xFFFF0000u), acc[u][2 * q + 1]);
         }
       }
     }
-    const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
-    const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
-    uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c8 * 8);
-    *dst = make_uint4(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv),
-                      pack_bf16(acc[4] * inv, acc[5] * inv), pack_bf16(acc[6] * inv, acc[7] * inv));
-    if (c8 == 0 && a.lse_out) a.lse_out[orow] = (M == NEG_INF) ? M : (M + log2f(Ls)) * kLn2;
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int item = base + u * kThreads;
+      if (item >= total) continue;
+      const int ur = item % rows, c8 = item / rows;
+      const int rg = rb * a.unit_rows + ur;
+      const int uu = rg / G, g = rg % G;
+      if (uu >= n) continue;
+      const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
+      uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c8 * 8);
+      *dst = make_uint4(pack_bf16(acc[u][0], acc[u][1]), pack_bf16(acc[u][2], acc[u][3]),
+                        pack_bf16(acc[u][4], acc[u][5]), pack_bf16(acc[u][6], acc[u][7]));
+    }
   }
 }
 
@@ -467,7 +491,7 @@ __global__ void __maxnreg__(168)
   if (a.lpt) {
     long long slot = blockIdx.x;
     if (a.B <= kLptMaxTrees) {
-      lpt_item(a, G, slot, reinterpret_cast<int*>(anc_s), misc);
+      lpt_item(a, G, slot, L::kMaxChunks, reinterpret_cast<int*>(anc_s), misc);
       b = misc[0];
       h = misc[1];
       rb = misc[2];
@@ -920,7 +944,9 @@ __global__ void __maxnreg__(168)
   if (*misc_last == 0) return;
   const char* slabs = static_cast<const char*>(a.ws) + a.slab_off +
                       (size_t)(slab - chunk) * L::kSlabBytes;
-  merge_chunks<D>(slabs, nch, rows, rb, G, n, off, h, a);
+  // the chunks' row weights go over the Q / K / V tiles, idle now (a split
+  // unit never stages its output there); lpt_item keeps nch within them
+  merge_chunks<D>(slabs, nch, rows, rb, G, n, off, h, reinterpret_cast<float*>(smem + L::kOffQ), a);
 }
 
 template <int D>
