@@ -288,87 +288,93 @@ __device__ void lpt_item(const AttnArgs& a, int G, long long slot, int max_chunk
 // (Sec. 3.1 attention as a softmax over the union of the chunks' keys).
 // Chunk s holds O_s / l_s (bf16), its max m_s (base 2) and sum l_s: with
 // w_s = 2^(m_s - M) l_s, M = max_s m_s, the row is o = sum_s w_s (O_s / l_s)
-// / sum_s w_s and lse = ln 2 (M + log2 sum_s w_s).  First one thread per
-// row turns the chunks' (m_s, l_s) into normalised weights in shared memory
-// (`wgt`, nc x kRows floats over the CTA's idle tile buffers); then every
-// thread accumulates kU (row, 8-column group) items at a time, the loads of
-// all kU items of a chunk in flight together, so the merge costs a few L2
-// round trips per chunk rather than one per item.  Kept out of line:
-// inlined, its registers made the kernel spill.
+// / sum_s w_s and lse = ln 2 (M + log2 sum_s w_s).  One thread per row: it
+// turns the chunks' (m_s, l_s) into normalised weights, kept in its own
+// column of `wgt` (2 nc x kRows floats over the CTA's idle tile buffers, so
+// no barrier is needed), then accumulates its D / 8 column groups, kU groups
+// of kS chunks with their loads in flight together.  Slab reads are
+// coalesced across the warp's rows; no per-item index arithmetic.  Kept out
+// of line: inlined, its registers made the kernel spill.
 template <int D>
-__device__ __noinline__ void merge_chunks(const char* slabs, int nc, int rows, int rb, int G, int n,
-                                          int off, int h, float* wgt, const AttnArgs& a) {
+__device__ __noinline__ void merge_chunks(const char* __restrict__ slabs, int nc, int rows, int rb,
+                                          int G, int n, int off, int h, float* __restrict__ wgt,
+                                          const AttnArgs& a) {
   using L = Layout<D>;
   const float NEG_INF = __int_as_float(0xff800000);
   constexpr int CG = D / 8;
-  constexpr int kU = 4;
-  for (int ur = threadIdx.x; ur < rows; ur += kThreads) {
-    float M = NEG_INF;
-    for (int s = 0; s < nc; ++s) {
-      const float m = __ldcg(reinterpret_cast<const float*>(slabs + (size_t)s * L::kSlabBytes +
-                                                            L::kSlabM) + ur);
-      const float l = __ldcg(reinterpret_cast<const float*>(slabs + (size_t)s * L::kSlabBytes +
-                                                            L::kSlabL) + ur);
-      wgt[s * kRows + ur] = m;  // m and l parked, weighted below
-      wgt[(nc + s) * kRows + ur] = l;
-      M = fmaxf(M, m);
+  constexpr int kU = 8;   // column groups per pass
+  constexpr int kS = 2;   // chunks per pass
+  constexpr int kSB = 8;  // chunks whose (m, l) are loaded at once
+  static_assert(CG % kU == 0, "column groups per pass");
+  const int ur = threadIdx.x;
+  if (ur >= rows) return;
+  const int rg = rb * a.unit_rows + ur;
+  const int uu = rg / G, g = rg % G;
+  if (uu >= n) return;
+  float M = NEG_INF;
+  for (int s0 = 0; s0 < nc; s0 += kSB) {
+    float mv[kSB], lv[kSB];
+#pragma unroll
+    for (int j = 0; j < kSB; ++j) {
+      const char* src = slabs + (size_t)min(s0 + j, nc - 1) * L::kSlabBytes;
+      mv[j] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabM) + ur);
+      lv[j] = __ldcg(reinterpret_cast<const float*>(src + L::kSlabL) + ur);
     }
-    float Ls = 0.f;
-    for (int s = 0; s < nc; ++s) {
-      const float m = wgt[s * kRows + ur];
-      const float w = (m == NEG_INF) ? 0.f : ex2(m - M) * wgt[(nc + s) * kRows + ur];
-      wgt[s * kRows + ur] = w;
-      Ls += w;
+#pragma unroll
+    for (int j = 0; j < kSB; ++j) {
+      if (s0 + j < nc) {
+        wgt[(s0 + j) * kRows + ur] = mv[j];  // m and l parked, weighted below
+        wgt[(nc + s0 + j) * kRows + ur] = lv[j];
+        M = fmaxf(M, mv[j]);
+      }
     }
-    const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
-    for (int s = 0; s < nc; ++s) wgt[s * kRows + ur] *= inv;
-    const int rg = rb * a.unit_rows + ur;
-    const int uu = rg / G, g = rg % G;
-    if (uu < n && a.lse_out)
-      a.lse_out[(size_t)(off + uu) * a.Hq + (size_t)(h * G + g)] =
-          (M == NEG_INF || !(Ls > 0.f)) ? NEG_INF : (M + log2f(Ls)) * kLn2;
   }
-  __syncthreads();
-  const int total = rows * CG;
-  for (int base = threadIdx.x; base < total; base += kU * kThreads) {
+  float Ls = 0.f;
+  for (int s = 0; s < nc; ++s) {
+    const float m = wgt[s * kRows + ur];
+    const float w = (m == NEG_INF) ? 0.f : ex2(m - M) * wgt[(nc + s) * kRows + ur];
+    wgt[s * kRows + ur] = w;
+    Ls += w;
+  }
+  const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
+  const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
+  if (a.lse_out) a.lse_out[orow] = (M == NEG_INF || !(Ls > 0.f)) ? NEG_INF : (M + log2f(Ls)) * kLn2;
+  uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D);
+  for (int c0 = 0; c0 < CG; c0 += kU) {
     float acc[kU][8];
 #pragma unroll
     for (int u = 0; u < kU; ++u)
 #pragma unroll
       for (int q = 0; q < 8; ++q) acc[u][q] = 0.f;
-    for (int s = 0; s < nc; ++s) {
-      const uint4* o = reinterpret_cast<const uint4*>(slabs + (size_t)s * L::kSlabBytes);
-      uint4 ov[kU];
+    for (int s0 = 0; s0 < nc; s0 += kS) {
+      uint4 ov[kS][kU];
 #pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int item = min(base + u * kThreads, total - 1);
-        ov[u] = __ldcg(o + (size_t)(item / rows) * kRows + item % rows);  // row-fastest
+      for (int e = 0; e < kS; ++e) {
+        const uint4* o = reinterpret_cast<const uint4*>(
+                             slabs + (size_t)min(s0 + e, nc - 1) * L::kSlabBytes) +
+                         (size_t)c0 * kRows + ur;
+#pragma unroll
+        for (int u = 0; u < kU; ++u) ov[e][u] = __ldcg(o + u * kRows);
       }
 #pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int item = min(base + u * kThreads, total - 1);
-        const float w = wgt[s * kRows + item % rows];
-        const uint32_t wd[4] = {ov[u].x, ov[u].y, ov[u].z, ov[u].w};
+      for (int e = 0; e < kS; ++e) {
+        if (s0 + e >= nc) break;
+        const float w = wgt[(s0 + e) * kRows + ur] * inv;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          acc[u][2 * q] = fmaf(w, __uint_as_float(wd[q] << 16), acc[u][2 * q]);
-          acc[u][2 * q + 1] = fmaf(w, __uint_as_float(wd[q] & 0xFFFF0000u), acc[u][2 * q + 1]);
+        for (int u = 0; u < kU; ++u) {
+          const uint32_t wd[4] = {ov[e][u].x, ov[e][u].y, ov[e][u].z, ov[e][u].w};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            acc[u][2 * q] = fmaf(w, __uint_as_float(wd[q] << 16), acc[u][2 * q]);
+            acc[u][2 * q + 1] = fmaf(w, __uint_as_float(wd[q] & 0xFFFF0000u), acc[u][2 * q + 1]);
+          }
         }
       }
     }
 #pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const int item = base + u * kThreads;
-      if (item >= total) continue;
-      const int ur = item % rows, c8 = item / rows;
-      const int rg = rb * a.unit_rows + ur;
-      const int uu = rg / G, g = rg % G;
-      if (uu >= n) continue;
-      const size_t orow = (size_t)(off + uu) * a.Hq + (size_t)(h * G + g);
-      uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + orow * D + c8 * 8);
-      *dst = make_uint4(pack_bf16(acc[u][0], acc[u][1]), pack_bf16(acc[u][2], acc[u][3]),
-                        pack_bf16(acc[u][4], acc[u][5]), pack_bf16(acc[u][6], acc[u][7]));
-    }
+    for (int u = 0; u < kU; ++u)
+      dst[c0 + u] = make_uint4(pack_bf16(acc[u][0], acc[u][1]), pack_bf16(acc[u][2], acc[u][3]),
+                               pack_bf16(acc[u][4], acc[u][5]), pack_bf16(acc[u][6], acc[u][7]));
   }
 }
 
