@@ -188,10 +188,13 @@ __device__ void lpt_item(const AttnArgs& a, int G, long long slot, int max_chunk
   int* units = scratch + B;
   int* order = scratch + 2 * B;
   int* nch = scratch + 3 * B;
-  long long* wsum = reinterpret_cast<long long*>(misc + 8);
+  // W fits an int with room for 5 W: a batch's units hold at most 8 row
+  // blocks per kv-head, so W <= 8 B Hkv S_max / 128, and the K/V cache of
+  // B Hkv S_max rows of 256 bytes or more must fit in device memory
+  int* wsum = misc + 8;
   if (threadIdx.x == 0) *wsum = 0;
   __syncthreads();
-  long long w = 0;
+  int w = 0;
   for (int t = threadIdx.x; t < B; t += kThreads) {
     const int off = a.node_off[t];
     const int n = a.node_off[t + 1] - off;
@@ -200,24 +203,28 @@ __device__ void lpt_item(const AttnArgs& a, int G, long long slot, int max_chunk
                     off + n <= a.n_total;
     tiles[t] = ok ? (P + n + kBN - 1) / kBN : 0;
     units[t] = ok ? a.Hkv * ((G * n + a.unit_rows - 1) / a.unit_rows) : 1;
-    w += (long long)tiles[t] * units[t];
+    w += tiles[t] * units[t];
   }
-  if (w) atomicAdd(reinterpret_cast<unsigned long long*>(wsum), (unsigned long long)w);
+  if (w) atomicAdd(wsum, w);
   __syncthreads();
   // chunk length: a quarter above the balanced share W / resident, so that
   // units near the share stay whole (cutting them only adds merges and a
   // second wave) while the long ones are cut
-  const long long chunk =
-      a.ws ? max((long long)a.chunk_min, (5 * *wsum + 4ll * a.resident - 1) / (4ll * a.resident))
-           : (1ll << 40);
-  for (int t = threadIdx.x; t < B; t += kThreads)
-    nch[t] = tiles[t] > 0 ? (int)min((long long)max_chunks, (tiles[t] + chunk - 1) / chunk) : 1;
+  const int chunk =
+      a.ws ? max(a.chunk_min, (5 * *wsum + 4 * a.resident - 1) / (4 * a.resident)) : (1 << 30);
+  // nch per tree, and each tree's chunk length in place of its tile count
+  // (the ranking below compares lengths only)
+  for (int t = threadIdx.x; t < B; t += kThreads) {
+    const int nc = tiles[t] > 0 ? min(max_chunks, (tiles[t] + chunk - 1) / chunk) : 1;
+    nch[t] = nc;
+    tiles[t] = (tiles[t] + nc - 1) / nc;
+  }
   __syncthreads();
   for (int t = threadIdx.x; t < B; t += kThreads) {
-    const int mine = (tiles[t] + nch[t] - 1) / nch[t];
+    const int mine = tiles[t];
     int rank = 0;
     for (int j = 0; j < B; ++j) {
-      const int o = (tiles[j] + nch[j] - 1) / nch[j];
+      const int o = tiles[j];
       rank += (o > mine || (o == mine && j < t)) ? 1 : 0;
     }
     order[rank] = t;

@@ -589,15 +589,18 @@ def test_tree_attn_serving_sweep(dev, B):
                                    atol=LSE_ABS, rtol=0)
 
 
-def test_tree_attn_long_tree_cut_into_key_chunks(dev):
+@pytest.mark.parametrize("p_long", [8000, 20000])
+def test_tree_attn_long_tree_cut_into_key_chunks(dev, p_long):
     """One long tree among short ones: the batch runs as whole units dealt
     longest first, and the long tree's units are cut into key chunks (about
     one resident CTA's share of the batch each) whose last one to finish
-    merges them.  The long tree and a short one carry random K/V and are
-    checked against the oracle; the others have all-zero K/V (outputs exactly
-    0, lse = ln of the number of keys each node sees).  Two calls in a row on
-    the same workspace: the chunk tickets are back at zero after each."""
-    P = [8000, 300, 500, 700, 900, 1100, 1300, 1500, 1700]
+    merges them (about 7 chunks for the 8000-token prefix, 11 for 20000: the
+    merge then takes its chunks' statistics in two batches).  The long tree
+    and a short one carry random K/V and are checked against the oracle; the
+    others have all-zero K/V (outputs exactly 0, lse = ln of the number of
+    keys each node sees).  Two calls in a row on the same workspace: the
+    chunk tickets are back at zero after each."""
+    P = [p_long, 300, 500, 700, 900, 1100, 1300, 1500, 1700]
     n = [64, 40, 48, 56, 64, 72, 80, 88, 96]
     shape = _attn_shape(len(P), P, n, [6] * len(P), 32, 8, 128, cap=10)
     drawn = [0, 4]
