@@ -74,6 +74,10 @@ __global__ void __launch_bounds__(kThreads, 1) global_prune_kernel(PruneArgs a) 
     if (v == 0) raise_status(a.status, kStTree);
     return;
   }
+  // rows outside every tree (node_off[0] > 0 or node_off[B] < n_total)
+  // belong to no result; the trees themselves are still pruned
+  if (v == 0 && ((b == 0 && off != 0) || (b == a.B - 1 && off + n != a.n_total)))
+    raise_status(a.status, kStTree);
   // ---- tree, validation, depth
   int p = -1;
   float s = 0.f;

@@ -30,12 +30,17 @@ __global__ void __launch_bounds__(kThreads) rescore_select_kernel(RescoreArgs a)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   pdl_launch_dependents();
   pdl_wait();
-  const int off = a.node_off[b];
-  const int n = a.node_off[b + 1] - off;
+  const int o_lo = a.node_off[b], o_hi = a.node_off[b + 1];
+  const int off = o_lo;
+  const int n = o_hi - o_lo;
   if (n < 1 || n > 256 || off < 0 || off + n > a.n_total) {
     if (tid == 0) raise_status(a.status, kStTree);
     return;
   }
+  // rows outside every tree (node_off[0] > 0 or node_off[B] < n_total)
+  // belong to no result; the trees themselves are still computed
+  if (tid == 0 && ((b == 0 && o_lo != 0) || (b == a.B - 1 && o_hi != a.n_total)))
+    raise_status(a.status, kStTree);
   const int v = tid;
   // every per-node input is requested at once; only the strong-row gather
   // depends on them (parent and token)

@@ -528,7 +528,8 @@ __global__ void __maxnreg__(168)
     P = a.prefix_len[b];
   }
   const bool bad_shape = !no_unit && (n < 1 || n > 256 || P < 0 || P + n > a.S_max || off < 0 ||
-                                      off + n > a.n_total || (b == 0 && off != 0));
+                                      off + n > a.n_total || (b == 0 && off != 0) ||
+                                      (b == a.B - 1 && off + n != a.n_total));
   const int rows = no_unit || bad_shape ? 0 : min(a.unit_rows, G * n - rb * a.unit_rows);
   const bool skip = rows <= 0;
   const bool two = rows > kBM;  // query tile 1 holds rows

@@ -373,7 +373,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---- shape checks (uniform over the cluster)
   const bool bad_shape = (n < 1 || n > 256 || P < 0 || P + n > a.S_max || off < 0 ||
-                          off + n > a.n_total || (b == 0 && off != 0));
+                          off + n > a.n_total || (b == 0 && off != 0) ||
+                          (b == a.B - 1 && off + n != a.n_total));
   const bool skip = bad_shape || r0 >= G * n;
   const int Lk = P + n;
   const int T = (Lk + kBN - 1) / kBN;

@@ -118,6 +118,29 @@ def test_tree_attn_llama70b_shape_sampled(dev):
         _check_attn(wl, o[a:e], lse[a:e], ref_o, ref_lse)
 
 
+@pytest.mark.parametrize("name", ["llama3-8b-verify", "llama3-70b-verify"])
+def test_tree_attn_rows_outside_every_tree_set_status(dev, name):
+    """node_off whose last entry falls short of n_total (rows in no tree) sets
+    TG_ERR_DEVICE_TREE, in the split kernel (one tree) and in the whole-unit
+    kernel (a batch), and the next well-formed call is exact."""
+    wl = synth.make_workload(name, seed=12, with_logits=False, with_strong=False)
+    short = wl["node_off"].copy()
+    short[-1] -= 3
+    q = _dev.bf16(wl["q"], dev)
+    k, v = _dev.bf16(wl["k_cache"], dev), _dev.bf16(wl["v_cache"], dev)
+    tg.tree_attn(q, k, v, _dev.i32(wl["prefix_len"], dev), _dev.i32(wl["parent"], dev),
+                 _dev.i32(short, dev), _dev.max_nodes(wl))
+    assert tg.last_device_status() & 4
+    o, lse = _run_attn(wl, dev)
+    off = wl["node_off"]
+    b = len(off) - 2                      # the last tree, the one the short extent cut
+    a, e = int(off[b]), int(off[b + 1])
+    ref_o, ref_lse = O.tree_attention(wl["q"][a:e], wl["k_cache"][b:b + 1], wl["v_cache"][b:b + 1],
+                                      wl["prefix_len"][b:b + 1], wl["parent"][a:e], [0, e - a],
+                                      Hkv=wl["shape"]["Hkv"])
+    _check_attn(wl, o[a:e], lse[a:e], ref_o, ref_lse)
+
+
 def test_tree_attn_malformed_tree_sets_status(dev):
     wl = synth.make_workload(_attn_shape(1, 16, 8, 3, 8, 8, 64), seed=4, with_logits=False,
                              with_strong=False)
@@ -274,6 +297,27 @@ def test_rescore_select_bit_exact(dev, name, visited):
     got = _run_rescore(wl, N, dev, vis)
     ref = O.rescore_select(wl["weak_edge"], wl["strong_lp"], wl["parent"], wl["token"], vis,
                            wl["node_off"], N)
+    for g, r in zip(got, ref):
+        np.testing.assert_array_equal(g, r)
+
+
+@pytest.mark.parametrize("name", ["llama3-8b-verify", "llama3-70b-verify"])
+def test_rescore_select_rows_outside_every_tree_set_status(dev, name):
+    """node_off that leaves rows in no tree (node_off[B] < n_total) sets
+    TG_ERR_DEVICE_TREE (the trees within their own extents are still
+    computed), and the next well-formed call is exact."""
+    wl = synth.make_workload(name, seed=5, with_logits=False)
+    N = wl["shape"]["N"]
+    short = wl["node_off"].copy()
+    short[-1] -= 2
+    e, s, sel, ns = tg.rescore_select(_dev.f32(wl["weak_edge"], dev), _dev.f32(wl["strong_lp"], dev),
+                                      _dev.i32(wl["parent"], dev), _dev.i32(wl["token"], dev),
+                                      _dev.u8(wl["visited"], dev), _dev.i32(short, dev),
+                                      _dev.max_nodes(wl), N)
+    assert tg.last_device_status() & 4
+    got = _run_rescore(wl, N, dev)
+    ref = O.rescore_select(wl["weak_edge"], wl["strong_lp"], wl["parent"], wl["token"],
+                           wl["visited"], wl["node_off"], N)
     for g, r in zip(got, ref):
         np.testing.assert_array_equal(g, r)
 
@@ -734,6 +778,24 @@ def test_global_prune_largest_trees_and_budgets(dev):
     for budget in (1, 63, 255):
         got, ref = _run_prune(parents, scores, budget, 16, dev)
         _check_prune(got, ref)
+
+
+def test_global_prune_rows_outside_every_tree_set_status(dev):
+    """node_off[B] < n_total leaves rows in no tree: TG_ERR_DEVICE_TREE, and
+    the trees within their extents are still pruned exactly."""
+    rng = synth.make_rng(77)
+    pars = [synth.expansion_tree(rng, 4, 5, 5) for _ in range(2)]
+    parent = np.concatenate(pars).astype(np.int32)
+    score = np.concatenate([synth.path_scores(rng, p) for p in pars]).astype(np.float32)
+    off = np.array([0, len(pars[0]), len(parent)], np.int32)
+    short = off.copy()
+    short[-1] -= 2                      # tree 1 loses its last two nodes (still a valid tree)
+    got = tg.global_prune(_dev.f32(score, dev), _dev.i32(parent, dev), _dev.i32(short, dev),
+                          int(np.max(np.diff(off))), 12, 8)
+    assert tg.last_device_status() & 4
+    ref = O.global_prune(parent, score, short, 12, 8)
+    for g, r in zip(got[:2], ref[:2]):  # kept nodes and their counts, both trees
+        np.testing.assert_array_equal(g.cpu().numpy(), r)
 
 
 def test_global_prune_malformed_tree_sets_status(dev):
