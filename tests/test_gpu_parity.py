@@ -681,6 +681,47 @@ def test_tree_attn_long_tree_cut_into_key_chunks(dev, p_long):
                                        atol=LSE_ABS, rtol=0)
 
 
+@pytest.mark.parametrize("D,Hq,Hkv", [(64, 32, 8), (128, 8, 8), (128, 64, 8)])
+def test_tree_attn_whole_units_head_dims_and_groups(dev, D, Hq, Hkv):
+    """Batches that fill the GPU with whole units, at head size 64 and at
+    GQA groups of 1 and 8 (the serving tests use 128 and 4): units of one and
+    of two query tiles, and one long tree whose units are cut into key chunks.
+    Two trees carry random K/V and are checked against the oracle; the others
+    have all-zero K/V (outputs exactly 0, lse = ln of the keys each node
+    sees)."""
+    P = [12000, 700, 1500, 300, 900, 2100, 60, 1200, 500, 1800, 1000, 400]
+    n = [90, 120, 64, 200, 33, 150, 100, 128, 17, 180, 75, 140]
+    shape = _attn_shape(len(P), P, n, [6] * len(P), Hq, Hkv, D, cap=10)
+    drawn = [1, 2]
+    wl = synth.make_workload(shape, seed=41, with_logits=False, with_strong=False, kv_trees=drawn)
+    k, v = _serving_kv(wl, dev)
+    q = _dev.bf16(wl["q"], dev)
+    B = len(P)
+    ws = torch.zeros(tg.tree_attn_workspace_size(B, _dev.max_nodes(wl), Hq, Hkv, D),
+                     dtype=torch.uint8, device=dev)
+    lse = torch.full((q.shape[0], q.shape[1]), float("nan"), device=dev)
+    out, _ = tg.tree_attn(q, k, v, _dev.i32(wl["prefix_len"], dev), _dev.i32(wl["parent"], dev),
+                          _dev.i32(wl["node_off"], dev), _dev.max_nodes(wl), lse_out=lse, ws=ws)
+    _status_clean()
+    o = _dev.bf16_to_np(out)
+    lse = lse.cpu().numpy().astype(np.float64)
+    off = wl["node_off"]
+    for i, b in enumerate(drawn):
+        a, e = int(off[b]), int(off[b + 1])
+        ref_o, ref_lse = O.tree_attention(wl["q"][a:e], wl["k_cache"][i:i + 1], wl["v_cache"][i:i + 1],
+                                          wl["prefix_len"][b:b + 1], wl["parent"][a:e], [0, e - a],
+                                          Hkv=Hkv)
+        _check_attn(wl, o[a:e], lse[a:e], ref_o, ref_lse)
+    for b in range(B):
+        if b in drawn:
+            continue
+        a, e = int(off[b]), int(off[b + 1])
+        assert np.all(o[a:e] == 0.0)
+        count = int(wl["prefix_len"][b]) + O.node_depth(wl["parent"][a:e]) + 1
+        np.testing.assert_allclose(lse[a:e], np.log(count)[:, None] * np.ones((1, Hq)),
+                                   atol=LSE_ABS, rtol=0)
+
+
 def test_accept_serving_sweep(dev):
     """accept on an 8-tree ragged serving batch (n 32-256, depth 4-10) with
     bf16 target logits over 128256 tokens, bumps planted at +40 so that long
