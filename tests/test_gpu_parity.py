@@ -49,6 +49,10 @@ ATTN_CASES = {
     "ragged-b3": _attn_shape(3, [5, 300, 1000], [2, 64, 128], [1, 6, 8], 32, 8, 128, cap=10),
     "n31-n32": _attn_shape(2, [128, 256], [31, 32], [3, 4], 16, 8, 64),
     "g8-d64-b2": _attn_shape(2, [64, 200], [40, 50], [5, 6], 64, 8, 64, cap=10),
+    # head size 64 with the keys split over CTAs: cooperative (GQA) and cluster (MHA) paths
+    "split-d64-gqa": _attn_shape(1, 4000, 60, 6, 32, 8, 64),
+    "split-coop-d64": _attn_shape(1, 8000, 60, 6, 32, 8, 64),
+    "split-cluster-d64-mha": _attn_shape(1, 1500, 64, 7, 32, 32, 64),
     # one split over four query tiles of 128 rows: the 33-, 64- and 1-node
     # trees leave tiles with no rows, the 33-node tree one with four
     "ragged-b4-empty-tiles": _attn_shape(4, [300, 17, 1000, 5], [33, 100, 64, 1], [5, 7, 6, 1], 32, 8,
