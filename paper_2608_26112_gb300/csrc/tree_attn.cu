@@ -15,9 +15,10 @@
 //               S_t = Q_t K^T (M=128, N=128, K=D) and O_t += P_t V (M=128,
 //               N=D, K=128, P read from TMEM), bf16 in, fp32 accumulate,
 //               completion signalled by tcgen05.commit on mbarriers.  Pipe
-//               order per key tile i: PV0(i) PV1(i) S0(i+1) S1(i+1), so the
+//               order per key tile i: PV0(i) S0(i+1) PV1(i) S1(i+1), so the
 //               tensor pipe runs one tile's products while the other tile's
-//               softmax runs (a two-tile ping-pong);
+//               softmax runs (a two-tile ping-pong).  The whole warp runs the
+//               issue loop and one lane issues;
 //   warps 2..5  softmax of query tile 0, warps 6..9 of query tile 1: one
 //               thread per row (TMEM lane = row), so a row's max and sum
 //               never leave the thread.  A thread reads its 128 S values
@@ -586,7 +587,8 @@ __global__ void __maxnreg__(168)
     __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
-    if (lane == 0 && nt > 0) {
+    // the whole warp runs this loop; one elected lane issues (see tc_mma_f16)
+    if (nt > 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kBN, false);
       constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, true);
       // Operand descriptors as base + offset / 16: the start-address field
@@ -616,7 +618,7 @@ __global__ void __maxnreg__(168)
                         (kk > 0 || acc) ? 1u : 0u);
         tc_commit(bar(BAR_O_DONE + t));
       };
-      bool ok = mbar_wait(bar(BAR_Q_FULL), 0) && mbar_wait(bar(BAR_K_FULL), 0);
+      bool ok = mbar_wait_warp(bar(BAR_Q_FULL), 0) && mbar_wait_warp(bar(BAR_K_FULL), 0);
       if (ok) {
         tc_fence_after();
         issue_s(0, 0);
@@ -630,7 +632,7 @@ __global__ void __maxnreg__(168)
         const int st = it & 1, ph = it & 1;
         const bool nxt = it + 1 < nt;
         const int st2 = (it + 1) & 1;
-        ok = mbar_wait(bar(BAR_P_FULL), ph) && mbar_wait(bar(BAR_V_FULL + st), (it >> 1) & 1);
+        ok = mbar_wait_warp(bar(BAR_P_FULL), ph) && mbar_wait_warp(bar(BAR_V_FULL + st), (it >> 1) & 1);
         if (!ok) break;
         tc_fence_after();
         issue_pv(0, st, it > 0);
@@ -639,26 +641,26 @@ __global__ void __maxnreg__(168)
           // S_t(it+1) overwrites the TMEM columns PV_t(it) reads P_t(it) from:
           // it waits for that product (products with different accumulators
           // are not ordered)
-          ok = mbar_wait(bar(BAR_K_FULL + st2), ((it + 1) >> 1) & 1) && mbar_wait(bar(BAR_O_DONE), ph);
+          ok = mbar_wait_warp(bar(BAR_K_FULL + st2), ((it + 1) >> 1) & 1) && mbar_wait_warp(bar(BAR_O_DONE), ph);
           if (!ok) break;
           tc_fence_after();
           issue_s(0, st2);
           if (!two) tc_commit(bar(BAR_K_EMPTY + st2));
         }
         if (two) {
-          if (!(ok = mbar_wait(bar(BAR_P_FULL + 1), ph))) break;
+          if (!(ok = mbar_wait_warp(bar(BAR_P_FULL + 1), ph))) break;
           tc_fence_after();
           issue_pv(1, st, it > 0);
           tc_commit(bar(BAR_V_EMPTY + st));
           if (nxt) {
-            if (!(ok = mbar_wait(bar(BAR_O_DONE + 1), ph))) break;
+            if (!(ok = mbar_wait_warp(bar(BAR_O_DONE + 1), ph))) break;
             tc_fence_after();
             issue_s(1, st2);
             tc_commit(bar(BAR_K_EMPTY + st2));
           }
         }
       }
-      if (!ok) raise_status(a.status, kStTimeout);
+      if (!ok && lane == 0) raise_status(a.status, kStTimeout);
     }
     __syncwarp();
   } else {

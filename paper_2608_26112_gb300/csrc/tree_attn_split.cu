@@ -16,7 +16,8 @@
 //
 // Warp roles (320 threads, one CTA per SM):
 //   warp 0      TMA producer: K and V tiles into a 2-stage ring, Q once;
-//   warp 1      TMEM owner and MMA issuer: S = Q K^T (M=128, N=128, K=D) into
+//   warp 1      TMEM owner and MMA issuer (the whole warp runs the issue loop,
+//               one lane issues): S = Q K^T (M=128, N=128, K=D) into
 //               one of two TMEM buffers and O += P V (M=128, N=D, K=128) with
 //               P read from TMEM, bf16 in, fp32 accumulate, completion
 //               signalled by tcgen05.commit on mbarriers.  Pipe order S(0)
@@ -423,26 +424,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
-    if (lane == 0 && nt > 0) {
+    // the whole warp runs this loop; one elected lane issues (see tc_mma_f16)
+    if (nt > 0) {
       constexpr uint32_t kIdS = idesc_bf16_f32(kBM, kBN, false);
       constexpr uint32_t kIdO = idesc_bf16_f32(kBM, D, true);
       const uint32_t tmem_O = tmem + 256u;
       // Operand descriptors as base + offset / 16: the start-address field
       // (bits 0-13, 16-byte units) of a base descriptor plus the byte offset
-      // of the operand, exact while the address stays below 256 KB.  One
-      // thread issues every product, so the few integer ops per MMA instead
-      // of a full descriptor build keep the tensor pipe fed.
+      // of the operand, exact while the address stays below 256 KB: a few
+      // integer ops per MMA instead of a full descriptor build keep the
+      // tensor pipe fed.
       const uint64_t dq0 = smem_desc_sw128(q_base, 16, 1024);
       const uint64_t dk0 = smem_desc_sw128(k_base, 16, 1024);
       const uint64_t dv0 = smem_desc_sw128(v_base, kRegion, 1024);
-      bool ok = mbar_wait(bar(BAR_Q_FULL), 0);
+      bool ok = mbar_wait_warp(bar(BAR_Q_FULL), 0);
       for (int it = 0; ok && it <= nt; ++it) {
         if (it < nt) {
           // S buffer it&1 holds P(it-2): S(it) may overwrite it once PV(it-2)
           // is done (MMAs with different accumulators are not ordered)
           const int st = it & 1;
-          ok = mbar_wait(bar(BAR_K_FULL + st), (it >> 1) & 1);
-          if (ok && it >= 2) ok = mbar_wait(bar(BAR_O_DONE + st), ((it - 2) >> 1) & 1);
+          ok = mbar_wait_warp(bar(BAR_K_FULL + st), (it >> 1) & 1);
+          if (ok && it >= 2) ok = mbar_wait_warp(bar(BAR_O_DONE + st), ((it - 2) >> 1) & 1);
           if (!ok) break;
           tc_fence_after();
           const uint64_t dk = dk0 + (uint64_t)((st * L::kKVBytes) >> 4);
@@ -457,7 +459,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (it > 0) {
           const int jt = it - 1, sp = jt & 1;
-          ok = mbar_wait(bar(BAR_P_FULL), jt & 1) && mbar_wait(bar(BAR_V_FULL + sp), (jt >> 1) & 1);
+          ok = mbar_wait_warp(bar(BAR_P_FULL), jt & 1) && mbar_wait_warp(bar(BAR_V_FULL + sp), (jt >> 1) & 1);
           if (!ok) break;
           tc_fence_after();
           const uint64_t dv = dv0 + (uint64_t)((sp * L::kKVBytes) >> 4);
@@ -473,7 +475,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_commit(bar(BAR_V_EMPTY + sp));
         }
       }
-      if (!ok) raise_status(a.status, kStTimeout);
+      if (!ok && lane == 0) raise_status(a.status, kStTimeout);
     }
     __syncwarp();
   }
