@@ -100,18 +100,26 @@ struct Layout {
   static_assert(kSlabBytes % 16 == 0 && kSlabM % 16 == 0, "16-byte slab groups");
 };
 
+__device__ __forceinline__ uint32_t ld_shared_u32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
+  return v;
+}
 // 32 mask bits of one node for tree slots [b0, b0 + 32): slot < 0 is the
-// committed prefix (always visible), slots >= 256 are beyond any tree.
-__device__ __forceinline__ uint32_t mask_word(const uint32_t* anc, int b0) {
+// committed prefix (always visible), slots >= 256 are beyond any tree.  The
+// node's bitmask row is at shared-memory address `row`: one register, where
+// a generic pointer takes two and the softmax loop, at the register cap,
+// would spill one and reload it from local memory on the tree's tile.
+__device__ __forceinline__ uint32_t mask_word(uint32_t row, int b0) {
   if (b0 <= -32) return 0xFFFFFFFFu;
   if (b0 < 0) {
     const int k = -b0;
-    return (anc[0] << k) | ((1u << k) - 1u);
+    return (ld_shared_u32(row) << k) | ((1u << k) - 1u);
   }
   const int w = b0 >> 5, sh = b0 & 31;
   if (w >= kAncWords) return 0u;
-  const uint32_t lo = anc[w];
-  const uint32_t hi = (w + 1 < kAncWords) ? anc[w + 1] : 0u;
+  const uint32_t lo = ld_shared_u32(row + 4 * w);
+  const uint32_t hi = (w + 1 < kAncWords) ? ld_shared_u32(row + 4 * (w + 1)) : 0u;
   return sh ? ((lo >> sh) | (hi << (32 - sh))) : lo;
 }
 
@@ -459,6 +467,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (it > 0) {
           const int jt = it - 1, sp = jt & 1;
+          const int jkey0 = (split + jt * S_kv) * kBN;
+          if (jkey0 + kBN > Lk) {
+            // last tile of the sequence: V rows past the end may hold
+            // anything; the warp zeroes them while the softmax of the tile
+            // runs, so that 0-weight rows contribute exactly 0
+            if (!(ok = mbar_wait_warp(bar(BAR_V_FULL + sp), (jt >> 1) & 1))) break;
+            const int row0 = Lk - jkey0, chunks = (kBN - row0) * (D / 64) * 8;
+            for (int i = lane; i < chunks; i += 32) {
+              const int rr = row0 + i / ((D / 64) * 8), c = (i >> 3) % (D / 64), q = i & 7;
+              st_shared_v4(v_base + sp * L::kKVBytes + c * kRegion + rr * 128 + q * 16,
+                           make_uint4(0u, 0u, 0u, 0u));
+            }
+            fence_proxy_async_smem();  // the zeroed rows (generic stores) for the PV product
+            __syncwarp();
+          }
           ok = mbar_wait_warp(bar(BAR_P_FULL), jt & 1) && mbar_wait_warp(bar(BAR_V_FULL + sp), (jt >> 1) & 1);
           if (!ok) break;
           tc_fence_after();
@@ -488,30 +511,46 @@ __global__ void __launch_bounds__(kThreads, 1)
   const float sl2 = a.scale_log2;      // softmax scale * log2(e): scores in base 2
   if (warp >= 2) {
     // parent array, validation and ancestor bitmasks, while the first
-    // copies and products are in flight (row kBM stays zero)
+    // copies and products are in flight (row kBM, for rows past the tree,
+    // stays zero)
     int bad = 0;
     for (int v = sidx; v < n; v += kSoftmaxThreads) {
       const int p = a.parent[off + v];
       par_s[v] = p;
       bad |= (v == 0) ? (p != -1) : (p < 0 || p >= v);
     }
-    for (int i = sidx; i < (kBM + 1) * kAncWords; i += kSoftmaxThreads) anc_s[i] = 0u;
+    if (sidx < kAncWords) anc_s[kBM * kAncWords + sidx] = 0u;
     if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(bad_flag, 1);
     softmax_bar();
-    if (*bad_flag == 0) {
+    // Only a split whose tiles reach the tree's keys reads the bitmasks.
+    // Each node's bits gather in registers along its parent chain (the walk
+    // of Algorithm 3) and its row is stored once.  A malformed tree keeps
+    // every tree slot masked; its outputs are undefined.
+    if (nt > 0 && (split + (nt - 1) * S_kv + 1) * kBN > P) {
+      const bool good = *bad_flag == 0;
       const int tile_nodes = min(kBM / G, n - u_base);
       for (int t = sidx; t < tile_nodes; t += kSoftmaxThreads) {
+        uint32_t m[kAncWords - 1];
+#pragma unroll
+        for (int k = 0; k < kAncWords - 1; ++k) m[k] = 0u;
+        if (good)
+          for (int v = u_base + t; v >= 0; v = par_s[v]) {
+            const int wi = v >> 5;
+            const uint32_t bit = 1u << (v & 31);
+#pragma unroll
+            for (int k = 0; k < kAncWords - 1; ++k) m[k] |= (k == wi) ? bit : 0u;
+          }
         uint32_t* w = anc_s + t * kAncWords;
-        for (int v = u_base + t; v >= 0; v = par_s[v]) w[v >> 5] |= 1u << (v & 31);
+#pragma unroll
+        for (int k = 0; k < kAncWords - 1; ++k) w[k] = m[k];
+        w[kAncWords - 1] = 0u;
       }
-    } else if (sidx == 0 && split == 0) {
-      // a malformed tree keeps every tree slot masked; its outputs are undefined
-      raise_status(a.status, kStTree);
     }
+    if (sidx == 0 && split == 0 && *bad_flag != 0) raise_status(a.status, kStTree);
     softmax_bar();
 
     const int u = (r0 + r) / G;
-    const uint32_t* anc = anc_s + (u < n ? (u - u_base) : kBM) * kAncWords;
+    const uint32_t anc = smem_u32(anc_s + (u < n ? (u - u_base) : kBM) * kAncWords);
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     const uint32_t tmem_O = tmem + 256u;
     float m_run = NEG_INF, l_run = 0.f;  // m_run in raw score units
@@ -533,6 +572,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int st = it & 1;
       const int tile_key0 = (split + it * S_kv) * kBN;
       const int key0 = tile_key0 + half * 64;  // first key of this thread's columns
+      // the ancestor-mask words of this thread's tree columns, read from
+      // shared memory while S is still being computed
+      const bool tree_cols = key0 + 64 > P;
+      uint32_t mw0 = 0xFFFFFFFFu, mw1 = 0xFFFFFFFFu;
+      if (tree_cols) {
+        mw0 = mask_word(anc, key0 - P);
+        mw1 = mask_word(anc, key0 + 32 - P);
+      }
       float s[64];
       float mx = NEG_INF;
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_S_FULL + st), (it >> 1) & 1));
@@ -544,12 +591,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld32f(ts, *reinterpret_cast<float(*)[32]>(&s[0]));
         tmem_ld32f(ts + 32, *reinterpret_cast<float(*)[32]>(&s[32]));
         tc_wait_ld();
-        if (key0 + 64 > P) {
-          const uint32_t mw0 = mask_word(anc, key0 - P);
-          const uint32_t mw1 = mask_word(anc, key0 + 32 - P);
+        if (tree_cols) {
 #pragma unroll
           for (int c = 0; c < 64; ++c) {
-            const bool vis = (((c < 32) ? mw0 : mw1) >> (c & 31)) & 1u;
+            const bool vis = ((c < 32) ? mw0 : mw1) & (1u << (c & 31));
             s[c] = vis ? s[c] : NEG_INF;
           }
         }
@@ -600,18 +645,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_wait_st();
         }
       }
-      if (tile_key0 + kBN > Lk) {
-        // last tile of the sequence: V rows past the end may hold anything;
-        // zero them so that 0-weight rows contribute exactly 0
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(BAR_V_FULL + st), (it >> 1) & 1));
-        if (!ok) continue;
-        if (tile_key0 + r >= Lk && half < D / 64) {
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            st_shared_v4(v_base + st * L::kKVBytes + half * kRegion + r * 128 + q * 16,
-                         make_uint4(0u, 0u, 0u, 0u));
-        }
-      }
       // this thread's 64 P values as bf16 pairs over its half of the S
       // buffer: columns st*128 + half*32 .. +32 (both halves have read their
       // S past the row-max barrier above)
@@ -622,7 +655,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_st32(tmem + (uint32_t)(st * 128 + half * 32) + lane_off, pw);
         tc_wait_st();
       }
-      fence_proxy_async_smem();  // the zeroed V rows (generic stores) for the PV product
       tc_fence_before();
       mbar_arrive(bar(BAR_P_FULL));
       m_run = m_new;
