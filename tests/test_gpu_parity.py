@@ -98,6 +98,18 @@ def test_tree_attn_ignores_nan_past_the_sequence(dev):
     _check_attn(wl, o, lse, ref_o, ref_lse)
 
 
+def test_tree_attn_whole_units_ignore_nan_past_the_sequence(dev):
+    # 2 trees x 8 kv-heads x 10 row tiles of 128 (G 8, 160 nodes) fill a wave
+    # of 152 SMs, so the whole-unit kernel runs; KV rows past each sequence
+    # hold NaN, and each sequence ends inside a key tile
+    wl = synth.make_workload(_attn_shape(2, [300, 517], [160, 100], [7, 6], 64, 8, 128, cap=16),
+                             seed=4, kv_tail="nan", with_logits=False, with_strong=False, S_max=800)
+    o, lse = _run_attn(wl, dev)
+    ref_o, ref_lse = O.tree_attention(wl["q"], wl["k_cache"], wl["v_cache"], wl["prefix_len"],
+                                      wl["parent"], wl["node_off"], Hkv=8)
+    _check_attn(wl, o, lse, ref_o, ref_lse)
+
+
 def test_tree_attn_chain_equals_causal(dev):
     # chain tree: the kernel's result must equal causal attention (oracle pin)
     shape = _attn_shape(1, 200, 40, 39, 32, 8, 128)
