@@ -98,6 +98,18 @@ def test_tree_attn_ignores_nan_past_the_sequence(dev):
     _check_attn(wl, o, lse, ref_o, ref_lse)
 
 
+def test_tree_attn_split_kernel_nan_one_row_into_the_last_tile(dev):
+    # one tree, keys 1000 + 25 = 1025: the last key tile holds one real row,
+    # so 127 V rows past the end (NaN here) are zeroed before its PV product,
+    # in a launch whose keys are split over several CTAs
+    wl = synth.make_workload(_attn_shape(1, 1000, 25, 5, 32, 8, 128), seed=5, kv_tail="nan",
+                             with_logits=False, with_strong=False, S_max=1200)
+    o, lse = _run_attn(wl, dev)
+    ref_o, ref_lse = O.tree_attention(wl["q"], wl["k_cache"], wl["v_cache"], wl["prefix_len"],
+                                      wl["parent"], wl["node_off"], Hkv=8)
+    _check_attn(wl, o, lse, ref_o, ref_lse)
+
+
 def test_tree_attn_whole_units_ignore_nan_past_the_sequence(dev):
     # 2 trees x 8 kv-heads x 10 row tiles of 128 (G 8, 160 nodes) fill a wave
     # of 152 SMs, so the whole-unit kernel runs; KV rows past each sequence
