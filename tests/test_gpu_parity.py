@@ -772,6 +772,67 @@ def test_accept_serving_sweep(dev):
     assert ref[1].max() >= 2
 
 
+def test_expand_topk_many_rows_llama_vocab(dev):
+    """336 bf16 rows over 128256 tokens picked by row_idx from 400 (k = 10):
+    two rows or more per SM, so whole rows are streamed by one CTA each (8
+    batches per row)."""
+    rng = synth.make_rng(21)
+    lg = synth.f32_to_bf16_bits(synth.normal_f32(rng, (400, 128256), 3.0))
+    rows = synth.make_rng(22).permutation(400)[:336].astype(np.int32)
+    ps = -np.abs(synth.normal_f32(rng, (336,), 4.0))
+    got = _run_expand(_dev.bf16(lg, dev), ps, 10, dev, row_idx=rows)
+    ref = O.expand_topk(lg, ps, 10, row_idx=rows, bf16=True)
+    _check_expand(got, ref)
+
+
+@pytest.mark.parametrize("V,ld,dtype,k", [(32001, 32008, "bf16", 32), (1023, 1024, "f32", 5),
+                                          (40000, 40000, "f32", 16)])
+def test_expand_topk_many_rows_ragged_vocab(dev, V, ld, dtype, k):
+    """320 rows, ragged vocabularies and row strides, both dtypes: the
+    streamed rows end inside a batch (or are shorter than one)."""
+    rng = synth.make_rng(V + 3 * k)
+    rows = 320
+    x = synth.normal_f32(rng, (rows, ld), 3.0)
+    ps = synth.normal_f32(rng, (rows,), 2.0)
+    if dtype == "bf16":
+        bits = synth.f32_to_bf16_bits(x)
+        got = _run_expand(_dev.bf16(bits, dev), ps, k, dev, V=V)
+        ref = O.expand_topk(bits[:, :V], ps, k, bf16=True)
+    else:
+        got = _run_expand(_dev.f32(x, dev), ps, k, dev, V=V)
+        ref = O.expand_topk(x[:, :V], ps, k)
+    _check_expand(got, ref)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_expand_topk_many_rows_ties_and_inf(dev, dtype):
+    """320 streamed rows of heavy ties (the candidate buffer overflows and the
+    exact-key fallback ranks the row), all -inf and signed-zero rows."""
+    rng = synth.make_rng(31)
+    rows, V = 320, 9000
+    x = rng.integers(-1, 2, size=(rows, V)).astype(np.float32)
+    x[7] = -np.inf
+    x[8, ::3] = -np.inf
+    x[9] = 0.0
+    x[10, :] = -0.0
+    x[10, 17] = 0.0
+    x[11, V - 1] = 0.5
+    x[100:200] = synth.normal_f32(rng, (100, V), 3.0)    # ordinary rows between
+    ps = synth.normal_f32(rng, (rows,), 1.0)
+    if dtype == "f32":
+        got = _run_expand(_dev.f32(x, dev), ps, 12, dev)
+        ref = O.expand_topk(x, ps, 12)
+    else:
+        bits = synth.f32_to_bf16_bits(x)
+        got = _run_expand(_dev.bf16(bits, dev), ps, 12, dev)
+        ref = O.expand_topk(bits, ps, 12, bf16=True)
+    np.testing.assert_array_equal(got[0], ref[0])
+    for g, r in zip(got[1:], ref[1:]):
+        np.testing.assert_array_equal(np.isneginf(g), np.isneginf(r))
+        fin = np.isfinite(r)
+        np.testing.assert_allclose(g[fin], r[fin], rtol=1e-5, atol=1e-5)
+
+
 def test_expand_topk_serving_rows(dev):
     """expand_topk over 128 frontier rows picked by row_idx from 512 bf16
     logit rows over 128256 tokens (k = 10), as a serving step expands the
